@@ -1,0 +1,181 @@
+"""Seeded synthetic workloads shared by the tests, the bench and the oracle checks.
+
+This module only describes shapes and draws random inputs; it holds none of the
+method's arithmetic (no quantisation, no dequantisation, no matmul), so that the
+CUDA path and the CPU oracle can both be fed from it without sharing code.
+
+The paper evaluates closed-loop policies whose weights and tasks are not
+available here (Section 4, Tables 3-4), so every input is synthetic: weights
+~N(0, 0.02) in fp32 (optionally with 1% of entries multiplied by 8), activations
+~N(0, 1) rounded to bf16.  The token counts follow one closed-loop step of the
+paper's batch-1 setting (Section 3.1 "Latency-first closed-loop control"):
+M=1 action-token decode, M=50 action-chunk denoising, M=280..816 prefix prefill.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+Q8_0 = 0
+Q4_0 = 1
+FMT_NAMES = {Q8_0: "Q8_0", Q4_0: "Q4_0"}
+
+
+@dataclasses.dataclass(frozen=True)
+class Linear:
+    """One weight matrix W [N][K] (PyTorch Linear.weight layout)."""
+    name: str
+    N: int
+    K: int
+    seed: int
+    outliers: float = 0.0  # fraction of weights multiplied by 8 before quantisation
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    fmt: int
+    M: int
+    layers: int
+    # linears of one layer, grouped by stage: the linears inside a group read the same
+    # activation (q/k/v, gate/up); a group only starts once the previous group is done.
+    groups: Sequence[Sequence[Linear]]
+    repeats: int = 1  # passes over the same weights (denoising steps)
+
+    def linears(self) -> List[Linear]:
+        return [lin for g in self.groups for lin in g]
+
+    @property
+    def params(self) -> int:
+        return sum(l.N * l.K for l in self.linears())
+
+    def weight_bytes(self) -> int:
+        per = 34 if self.fmt == Q8_0 else 18
+        return sum(l.N * l.K // 32 * per for l in self.linears())
+
+    def algorithmic_bytes(self) -> int:
+        """Weights read once + X read once (bf16) + Y written once (fp32), per pass."""
+        return self.weight_bytes() + sum(self.M * l.K * 2 + self.M * l.N * 4
+                                         for l in self.linears())
+
+    def flops(self) -> int:
+        return sum(2 * self.M * l.N * l.K for l in self.linears())
+
+
+def _decoder_layers(prefix: str, n_layers: int, hidden: int, kv: int, ffn: int,
+                    seed_base: int, outliers: float = 0.0, q: Optional[int] = None):
+    q = hidden if q is None else q
+    groups = []
+    for layer in range(n_layers):
+        s = seed_base + 16 * layer
+        groups.append([Linear(f"{prefix}{layer}.q", q, hidden, s + 0, outliers),
+                       Linear(f"{prefix}{layer}.k", kv, hidden, s + 1, outliers),
+                       Linear(f"{prefix}{layer}.v", kv, hidden, s + 2, outliers)])
+        groups.append([Linear(f"{prefix}{layer}.o", hidden, q, s + 3, outliers)])
+        groups.append([Linear(f"{prefix}{layer}.gate", ffn, hidden, s + 4, outliers),
+                       Linear(f"{prefix}{layer}.up", ffn, hidden, s + 5, outliers)])
+        groups.append([Linear(f"{prefix}{layer}.down", hidden, ffn, s + 6, outliers)])
+    return groups
+
+
+def _vit_layers(n_layers: int, width: int, mlp: int, seed_base: int):
+    groups = []
+    for layer in range(n_layers):
+        s = seed_base + 16 * layer
+        groups.append([Linear(f"vit{layer}.qkv", 3 * width, width, s + 0)])
+        groups.append([Linear(f"vit{layer}.o", width, width, s + 1)])
+        groups.append([Linear(f"vit{layer}.fc1", mlp, width, s + 2)])
+        groups.append([Linear(f"vit{layer}.fc2", width, mlp, s + 3)])
+    return groups
+
+
+def single_linear() -> Workload:
+    """One 2048x2048 Q8_0 linear at M=1."""
+    return Workload("single_q8_0_2048x2048_m1", Q8_0, 1, 1,
+                    [[Linear("w", 2048, 2048, 1)]])
+
+
+def gemma2b_decode(fmt: int) -> Workload:
+    """Gemma-style 2B decoder linears, 18 layers, hidden 2048, kv 256, ffn 16384, M=1."""
+    return Workload(f"gemma2b_decode_{FMT_NAMES[fmt].lower()}_m1", fmt, 1, 18,
+                    _flatten_layers(_decoder_layers("L", 18, 2048, 256, 16384, 1000)))
+
+
+def action_expert_denoise() -> Workload:
+    """Flow-matching action expert: 18 layers, width 1024, M=50, 10 denoising steps."""
+    return Workload("action_expert_q8_0_m50_x10", Q8_0, 50, 18,
+                    _flatten_layers(_decoder_layers("A", 18, 1024, 128, 4096, 3000)),
+                    repeats=10)
+
+
+def gemma2b_prefill(fmt: int) -> Workload:
+    """Backbone prefill over 3x256 image + 48 text tokens (M=816)."""
+    return Workload(f"gemma2b_prefill_{FMT_NAMES[fmt].lower()}_m816", fmt, 816, 18,
+                    _flatten_layers(_decoder_layers("L", 18, 2048, 256, 16384, 1000)))
+
+
+def vit_tower(fmt: int) -> Workload:
+    """ViT-style vision tower, width 1152, 27 layers, M=768."""
+    return Workload(f"vit_{FMT_NAMES[fmt].lower()}_m768", fmt, 768, 27,
+                    _flatten_layers(_vit_layers(27, 1152, 4608, 5000)))
+
+
+def llama7b(M: int) -> Workload:
+    """Llama-style 7B backbone, 32 layers, hidden 4096, ffn 11008, Q4_0 with 1% outliers."""
+    return Workload(f"llama7b_q4_0_m{M}", Q4_0, M, 32,
+                    _flatten_layers(_decoder_layers("L", 32, 4096, 4096, 11008, 7000,
+                                                    outliers=0.01)))
+
+
+def _flatten_layers(groups):
+    return tuple(tuple(g) for g in groups)
+
+
+def all_workloads() -> List[Workload]:
+    return [single_linear(), gemma2b_decode(Q8_0), gemma2b_decode(Q4_0),
+            action_expert_denoise(), gemma2b_prefill(Q8_0), gemma2b_prefill(Q4_0),
+            vit_tower(Q8_0), vit_tower(Q4_0), llama7b(1), llama7b(280)]
+
+
+# --------------------------------------------------------------------------- generators
+
+def weight_torch(lin: Linear, device="cpu"):
+    """fp32 W [N][K] ~ N(0, 0.02) from lin.seed (torch generator on `device`)."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(lin.seed)
+    w = torch.randn(lin.N, lin.K, generator=g, device=device, dtype=torch.float32) * 0.02
+    if lin.outliers > 0:
+        mask = torch.rand(lin.N, lin.K, generator=g, device=device) < lin.outliers
+        w = torch.where(mask, w * 8.0, w)
+    return w
+
+
+def activation_torch(M: int, K: int, seed: int, device="cpu"):
+    """bf16 X [M][K]: ~N(0, 1) drawn in fp32 and rounded to bf16 (round to nearest even)."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    return torch.randn(M, K, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+
+
+def activation_seed(lin: Linear, step: int = 0) -> int:
+    return 1_000_003 * (step + 1) + lin.seed
+
+
+def weight_np(N: int, K: int, seed: int, scale: float = 0.02) -> np.ndarray:
+    return (np.random.default_rng(seed).standard_normal((N, K)) * scale).astype(np.float32)
+
+
+def bf16_bits_np(x: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns of fp32 values via torch's conversion (input preparation only)."""
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(torch.bfloat16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def activation_bits_np(M: int, K: int, seed: int) -> np.ndarray:
+    x = np.random.default_rng(seed).standard_normal((M, K)).astype(np.float32)
+    return bf16_bits_np(x)
