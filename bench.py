@@ -1,0 +1,515 @@
+#!/usr/bin/env python3
+"""Benchmark of the block-quantised matmul hot path on GB300.
+
+Default workload (one "step"): the action-token decode of a Gemma-style 2B backbone
+at M=1 -- 18 layers x (q, k, v, o, gate, up, down) linears -- once with Q8_0 and once
+with Q4_0 weights, each chain replayed as a CUDA graph of emb_qlayer_seq (fused
+q/k/v and gate/up launches, programmatic dependent launch between launches). This is
+the paper's latency-first batch-1 execution (Section 3.1 challenge 2, Section 3.2
+principle 2) on its 8-bit / 4-bit configurations (Section 4, Table 3).
+
+Metric: algorithmic HBM bytes (packed weights read once + bf16 X + fp32 Y) per second,
+i.e. GB/s against the HBM roofline; for --workload with M >= 50 it is TFLOP/s against
+the bf16 tensor-core roofline.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload NAME]
+
+N > 1: one process per GPU (torchrun); every rank runs its own replica of the step
+(weak scaling, no collective on the data path); time = max over ranks.
+--impl reference: the CPU oracle timed on the host cores on a bounded sample of the
+same workload (this build has no other reference implementation).
+"""
+from __future__ import annotations
+
+import argparse
+import concurrent.futures as cf
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
+BAD_CLOCK_REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown")
+
+
+# ------------------------------------------------------------------ helpers
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def init_dist(world: int, backend: str):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+    return dist if world > 1 else None
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(value: float, dist, device=None) -> float:
+    """Largest value across ranks (the slowest rank sets the whole-job time)."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, dist, device=None) -> float:
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            p = json.load(fh)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": FALLBACK_HBM_GBS, "bf16_tflops": FALLBACK_BF16_TFLOPS,
+                "bf16_tflops_sustained": FALLBACK_BF16_TFLOPS_SUSTAINED, "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu), "-lms", "200"], stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.flush()
+        self.out.seek(0)
+        rows = [ln.strip().split(", ") for ln in self.out.read().splitlines() if ln.strip()]
+        self.out.close()
+        os.unlink(self.out.name)
+        return summarize_clocks(rows)
+
+
+def summarize_clocks(rows):
+    names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+    sm, mx, reasons, power = [], None, set(), []
+    for r in rows:
+        if len(r) < 9:
+            continue
+        try:
+            sm.append(float(r[1]))
+            mx = float(r[2])
+            power.append(float(r[3]))
+        except ValueError:
+            continue
+        for name, val in zip(names, r[5:9]):
+            if val.strip().lower() == "active":
+                reasons.add(name)
+    if not sm:
+        return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": ["no samples"]}
+    # samples under load: the timed region keeps the GPU busy; drop idle-clock samples
+    loaded = [v for v in sm if v >= 0.5 * max(sm)] or sm
+    return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx, "reasons": sorted(reasons),
+            "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+# ------------------------------------------------------------------ workloads
+
+WORKLOADS = {
+    "gemma2b_decode": lambda: [wl.gemma2b_decode(wl.Q8_0), wl.gemma2b_decode(wl.Q4_0)],
+    "single_linear": lambda: [wl.single_linear()],
+    "action_expert": lambda: [wl.action_expert_denoise()],
+    "gemma2b_prefill": lambda: [wl.gemma2b_prefill(wl.Q8_0), wl.gemma2b_prefill(wl.Q4_0)],
+    "vit": lambda: [wl.vit_tower(wl.Q8_0), wl.vit_tower(wl.Q4_0)],
+    "llama7b_decode": lambda: [wl.llama7b(1)],
+    "llama7b_prefill": lambda: [wl.llama7b(280)],
+}
+
+
+def build_chain(w: wl.Workload, device):
+    """Device weights (generated, quantised, fp32 freed), activations and outputs."""
+    import torch
+    import paper_2607_02501_gb300 as emb
+    specs, xs, ys = [], [], []
+    for group in w.groups:
+        K = group[0].K
+        X = wl.activation_torch(w.M, K, wl.activation_seed(group[0]), device=device)
+        xs.append(X)
+        for lin in group:
+            W = wl.weight_torch(lin, device=device)
+            img = emb.quantize(w.fmt, W)
+            del W
+            Y = torch.empty(w.M, lin.N, dtype=torch.float32, device=device)
+            ys.append(Y)
+            specs.append((w.fmt, img, lin.N, lin.K, X, Y))
+    torch.cuda.synchronize()
+    return specs, xs, ys
+
+
+def count_launches(specs) -> int:
+    """Kernel launches of one emb_qlayer_seq over these layers (fused groups)."""
+    n, prev = 0, None
+    size = 0
+    for sp in specs:
+        key = (sp[0], sp[3], sp[4].data_ptr())
+        if key == prev and size < 4:
+            size += 1
+            continue
+        n += 1
+        prev, size = key, 1
+    return n
+
+
+def capture_graph(specs, M):
+    import torch
+    import paper_2607_02501_gb300 as emb
+    layers = emb.make_layers(specs)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        emb.emb_qlayer_seq(layers, M)      # first call: module load, tensor-map setup
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        emb.emb_qlayer_seq(layers, M)
+    torch.cuda.synchronize()
+    return g, layers
+
+
+# ------------------------------------------------------------------ CPU oracle timing
+
+def oracle_sample_images(w: wl.Workload, layers: int):
+    """Host-side packed images (made by the oracle) for the first `layers` layers."""
+    import oracle
+    import torch
+    lins = [lin for g in w.groups[:4 * layers] for lin in g]
+
+    def one(lin):
+        W = wl.weight_torch(lin, device="cpu").numpy()
+        return lin, oracle.quantize(w.fmt, W)
+
+    with cf.ThreadPoolExecutor(max_workers=max(1, oracle.host_threads())) as ex:
+        imgs = list(ex.map(one, lins))
+    xs = {}
+    for g in w.groups[:4 * layers]:
+        X = wl.activation_torch(w.M, g[0].K, wl.activation_seed(g[0]), device="cpu")
+        bits = X.view(torch.int16).numpy().view("uint16")
+        for lin in g:
+            xs[lin.name] = bits
+    return [(lin, img, xs[lin.name]) for lin, img in imgs]
+
+
+def time_oracle(work, fmt, M, budget_s: float, min_rounds: int = 1):
+    """Run the oracle matmul over `work` (list of (lin, img, X)) repeatedly until
+    budget_s has passed; returns (bytes/s, elapsed, rounds)."""
+    import oracle
+    nbytes = 0
+    t0 = time.perf_counter()
+    rounds = 0
+    while True:
+        for lin, img, X in work:
+            oracle.qmatmul(fmt, img, X, lin.N, lin.K)
+            nbytes += lin.N * lin.K // 32 * (34 if fmt == wl.Q8_0 else 18) + M * lin.K * 2 + M * lin.N * 4
+        rounds += 1
+        el = time.perf_counter() - t0
+        if rounds >= min_rounds and el >= budget_s:
+            return nbytes / el, el, rounds
+
+
+def cpu_baseline(workloads, budget_s=8.0, layers=2):
+    import oracle
+    threads = oracle.host_threads()
+    total_bytes, total_t = 0.0, 0.0
+    for w in workloads:
+        work = oracle_sample_images(w, min(layers, w.layers))
+        bps, el, rounds = time_oracle(work, w.fmt, w.M, budget_s / len(workloads))
+        total_bytes += bps * el
+        total_t += el
+    sample = (f"first {layers} of {workloads[0].layers} layers "
+              f"({7 * layers} linears) per format, repeated over ~{budget_s:.0f} s; "
+              f"fp64 oracle matmul from oracle-packed weights, {threads} host threads")
+    return {"value": total_bytes / total_t / 1e9, "unit": "GB/s", "cores": threads,
+            "kind": "oracle", "sample": sample}
+
+
+# ------------------------------------------------------------------ arms
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    ws = WORKLOADS[args.workload]()
+    import oracle
+    oracle.build()
+    threads = oracle.host_threads()
+    # one step = the oracle over a fixed sample of linears (layer 0 of each format),
+    # sized so the whole run stays within a few minutes
+    work = [(w, oracle_sample_images(w, 1)) for w in ws]
+    per_step_target = min(1.0, 90.0 / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        for w, items in work:
+            time_oracle(items[:1], w.fmt, w.M, 0.0)
+    # pick how many linears a step covers from one calibration pass
+    t0 = time.perf_counter()
+    for w, items in work:
+        time_oracle(items[:1], w.fmt, w.M, 0.0)
+    one = (time.perf_counter() - t0) / len(work)
+    per_fmt = max(1, min(7, int(per_step_target / max(one, 1e-6) / len(work))))
+    nbytes = 0
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for w, items in work:
+            for lin, img, X in items[:per_fmt]:
+                oracle.qmatmul(w.fmt, img, X, lin.N, lin.K)
+                nbytes += (lin.N * lin.K // 32 * (34 if w.fmt == wl.Q8_0 else 18)
+                           + w.M * lin.K * 2 + w.M * lin.N * 4)
+    el = time.perf_counter() - t0
+    value = nbytes / el / 1e9
+    sample = (f"each step: the fp64 oracle over the first {per_fmt} linears of layer 0 "
+              f"per format ({threads} host threads)")
+    line = {"impl": "reference", "metric": metric_name(ws), "value": value, "unit": "GB/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": el / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_of(ws, args),
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": threads,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def metric_name(ws) -> str:
+    return "qmatmul µs & HBM GB/s (M=1) / TFLOP/s (M≥50), as fraction of roofline"
+
+
+def config_of(ws, args):
+    w0 = ws[0]
+    return {"workload": args.workload,
+            "formats": [wl.FMT_NAMES[w.fmt] for w in ws],
+            "M": w0.M, "layers": w0.layers, "linears_per_format": len(w0.linears()),
+            "repeats": w0.repeats,
+            "weight_bytes_per_step": sum(w.weight_bytes() * w.repeats for w in ws),
+            "l2": "inputs larger than L2 (weights per step >> 126 MB L2)"
+            if sum(w.weight_bytes() for w in ws) > 400e6 else "weights rotate through L2",
+            "parallelism": f"replica x{int(os.environ.get('WORLD_SIZE', '1'))}"}
+
+
+def run_ours(args):
+    import torch
+    import paper_2607_02501_gb300 as emb
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = init_dist(world, "nccl")
+    emb.lib()
+    ws = WORKLOADS[args.workload]()
+    chains = []
+    for w in ws:
+        specs, xs, ys = build_chain(w, dev)
+        g, layers = capture_graph(specs, w.M)
+        chains.append({"w": w, "specs": specs, "xs": xs, "ys": ys, "graph": g, "layers": layers,
+                       "launches": count_launches(specs),
+                       "bytes": w.algorithmic_bytes(), "flops": w.flops()})
+    tensor_bound = ws[0].M >= 50
+    # warm-up
+    for _ in range(args.warmup):
+        for c in chains:
+            for _ in range(c["w"].repeats):
+                c["graph"].replay()
+    torch.cuda.synchronize()
+    assert emb.emb_device_status() == emb.EMB_OK
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(chains) + 1)]
+          for _ in range(args.steps)]
+    barrier(dist)
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        ev[i][0].record()
+        for j, c in enumerate(chains):
+            for _ in range(c["w"].repeats):
+                c["graph"].replay()
+            ev[i][j + 1].record()
+    torch.cuda.synchronize()
+    barrier(dist)
+    clocks = sampler.stop()
+    total_ms = ev[0][0].elapsed_time(ev[-1][-1])
+    chain_ms = [sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(args.steps))
+                for j in range(len(chains))]
+    assert emb.emb_device_status() == emb.EMB_OK
+    max_ms = max_over_ranks(total_ms, dist, dev)
+
+    step_bytes = sum(c["bytes"] * c["w"].repeats for c in chains)
+    step_flops = sum(c["flops"] * c["w"].repeats for c in chains)
+    if tensor_bound:
+        value = world * step_flops * args.steps / (max_ms / 1e3) / 1e12
+        unit = "TFLOP/s"
+    else:
+        value = world * step_bytes * args.steps / (max_ms / 1e3) / 1e9
+        unit = "GB/s"
+
+    # dominant kernel family: the chain that takes the most time
+    peaks = load_peaks()
+    j = max(range(len(chains)), key=lambda k: chain_ms[k])
+    c = chains[j]
+    launches = c["launches"] * c["w"].repeats * args.steps
+    per_launch_ms = chain_ms[j] / launches
+    if tensor_bound:
+        achieved = c["flops"] * c["w"].repeats * args.steps / launches / (per_launch_ms / 1e3) / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops_sustained"],
+                "unit": "TFLOP/s", "peak_source": f"{peaks['source']} bf16 dense (sustained)"}
+    else:
+        achieved = c["bytes"] * c["w"].repeats * args.steps / launches / (per_launch_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "peak_source": f"{peaks['source']} HBM copy bandwidth"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = kernel_traffic(args.workload, c["w"])
+    roof["kernel"] = ("gemv_kernel" if c["w"].M <= 4 else "gemm_tc_kernel") + \
+        f"<{wl.FMT_NAMES[c['w'].fmt]}>"
+    roof["launches_per_step"] = c["launches"] * c["w"].repeats
+    roof["per_launch_us"] = per_launch_ms * 1e3
+
+    e2e = measure_e2e(chains, args, dev, dist, tensor_bound)
+
+    gpu_launches = sum(cc["launches"] * cc["w"].repeats for cc in chains) * args.steps
+    line = {"metric": metric_name(ws), "value": value, "unit": unit, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": max_ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if tensor_bound else "f32", "data": "synthetic",
+            "config": config_of(ws, args), "roofline": roof, "e2e": e2e, "clocks": clocks,
+            "gpu_launches": gpu_launches,
+            "per_format": {wl.FMT_NAMES[cc["w"].fmt]: {
+                "ms_per_step": chain_ms[k] / args.steps,
+                ("TFLOP/s" if tensor_bound else "GB/s"):
+                    (cc["flops"] if tensor_bound else cc["bytes"]) * cc["w"].repeats * args.steps
+                    / (chain_ms[k] / 1e3) / (1e12 if tensor_bound else 1e9)}
+                for k, cc in enumerate(chains)}}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        torch.cuda.synchronize()
+        line["cpu_baseline"] = cpu_baseline(ws)
+    if rank == 0:
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def kernel_traffic(workload, w):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu summary, if
+    one exists for this workload and matches the current kernel build."""
+    path = os.path.join(ROOT, "profiles", f"traffic_{workload}.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        return d.get(wl.FMT_NAMES[w.fmt])
+    except (OSError, ValueError):
+        return None
+
+
+def measure_e2e(chains, args, dev, dist, tensor_bound):
+    """Same metric through the public call a user makes: per step, copy every layer's
+    activations from pinned host memory, run emb_qlayer_seq for each format, copy every
+    output back, synchronise."""
+    import torch
+    import paper_2607_02501_gb300 as emb
+    host_x = [[x.cpu().pin_memory() for x in c["xs"]] for c in chains]
+    host_y = [[torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in c["ys"]] for c in chains]
+    h2d = sum(x.numel() * x.element_size() for hx in host_x for x in hx)
+    d2h = sum(y.numel() * y.element_size() for hy in host_y for y in hy)
+    steps = max(1, min(args.steps, 200))
+
+    def one_step():
+        for k, c in enumerate(chains):
+            for hx, x in zip(host_x[k], c["xs"]):
+                x.copy_(hx, non_blocking=True)
+            for _ in range(c["w"].repeats):
+                emb.emb_qlayer_seq(c["layers"], c["w"].M)
+            for hy, y in zip(host_y[k], c["ys"]):
+                hy.copy_(y, non_blocking=True)
+        torch.cuda.synchronize()
+
+    for _ in range(3):
+        one_step()
+    barrier(dist)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one_step()
+    el = max_over_ranks(time.perf_counter() - t0, dist, dev)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if tensor_bound:
+        work = sum(c["flops"] * c["w"].repeats for c in chains)
+        val, unit = world * work * steps / el / 1e12, "TFLOP/s"
+    else:
+        work = sum(c["bytes"] * c["w"].repeats for c in chains)
+        val, unit = world * work * steps / el / 1e9, "GB/s"
+    return {"value": val, "unit": unit, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": steps, "ms_per_step": el / steps * 1e3,
+            "how": "eager emb_qlayer_seq per format + pinned H2D of X / D2H of Y each step"}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="gemma2b_decode")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,176 @@
+/*
+ * emb_qmm.h -- C ABI of libembqmm.so, the GB300 (sm_103a) block-quantised
+ * weight x bf16 activation matmul that carries every linear layer of a
+ * vision-language-action backbone and action head in batch-1 embodied inference.
+ *
+ * Paper: "Embodied.cpp: A Portable Inference Runtime of Embodied AI Models on
+ * Heterogeneous Robots" (arXiv 2607.02501).
+ *   - batch-1, latency-first execution: Section 3.1, challenge 2
+ *     ("Latency-first closed-loop control"); Section 3.2, design principle 2
+ *     ("Latency-first fused execution": graph replay, buffer reuse, operator
+ *     fusion, careful host-device data movement);
+ *   - the 8-bit and 4-bit weight configurations: Section 4 ("VLA model
+ *     evaluation"), Table 3 columns "C++ 8-bit" / "C++ 4-bit";
+ *   - a stable deployment boundary behind one backend abstraction: abstract;
+ *     Section 3.2 (Figure 2 description).
+ * The paper gives no byte format; the two block formats below are this
+ * library's definition of the 8-bit and 4-bit configurations.
+ *
+ * Conventions for every entry point
+ *   - W is [N][K] (output features x input features, PyTorch Linear.weight
+ *     layout), X is [M][K] row-major bf16 (passed as its 16-bit patterns),
+ *     Y is [M][N] row-major fp32, and Y[m][n] = sum_k w'[n][k] * x[m][k].
+ *   - Every pointer argument is DEVICE memory owned by the caller, except the
+ *     `layers` array of emb_qlayer_seq, which is host memory read during the
+ *     call only. The library allocates nothing and keeps no per-call state; all
+ *     calls are reentrant and thread-safe.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) without any host synchronisation, except emb_device_status.
+ *   - Argument errors are reported BEFORE anything is enqueued. Launch errors
+ *     return EMB_ECUDA. Device-side failures (a bounded wait that expired) are
+ *     recorded in a device status word read by emb_device_status.
+ *   - Outputs are fully overwritten. Inputs and outputs must not overlap.
+ */
+#ifndef EMB_QMM_H
+#define EMB_QMM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define EMB_API __attribute__((visibility("default")))
+#else
+#define EMB_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t (the runtime's stream handle); NULL = default stream. */
+typedef struct CUstream_st* emb_stream_t;
+
+typedef enum {
+    /* 32 consecutive weights of one row along K share one fp16 scale d;
+     * each weight is an int8 code q in [-127, 127]; w' = d * q.
+     * d = fp16_rne(max|w| / 127), q = clamp(round_half_away(w / d), -127, 127). */
+    EMB_Q8_0 = 0,
+    /* 32 consecutive weights share one fp16 scale d; each weight is a 4-bit code
+     * q in [0, 15]; w' = d * (q - 8). With m the signed weight of largest
+     * magnitude (lowest index on ties): d = fp16_rne(m / -8),
+     * q = clamp(round_half_away(w / d), -8, 7) + 8. */
+    EMB_Q4_0 = 1
+} emb_qfmt;
+
+typedef enum {
+    EMB_OK = 0,
+    EMB_EINVAL = 1,        /* unknown format, M/N/K < 1, K % 32 != 0, NULL pointer,
+                              overlapping buffers, too many layers */
+    EMB_EALIGN = 2,        /* a device pointer is not 16-byte aligned
+                              (W_blocks must be 256-byte aligned) */
+    EMB_ENOSPC = 3,        /* workspace smaller than emb_qlayer_seq_workspace() */
+    EMB_ECUDA = 4,         /* a CUDA runtime call or launch failed */
+    EMB_ETIMEOUT = 5,      /* a device-side bounded wait expired (emb_device_status) */
+    EMB_EUNSUPPORTED = 6   /* shape outside what this build supports (see limits) */
+} emb_status;
+
+/* ---------------------------------------------------------------- packed weights
+ * Packed image of one [N][K] matrix (one caller allocation of
+ * emb_qweight_bytes(fmt, N, K) bytes, 256-byte aligned, written only by
+ * emb_quantize_*; callers may copy, save and reload it as plain bytes):
+ *   codes plane at byte 0:
+ *     Q8_0: int8  [N][K], row-major;
+ *     Q4_0: uint8 [N][K/2]; in each 32-weight block, byte j (0..15) holds
+ *           code j in its low nibble and code j+16 in its high nibble;
+ *   scales plane at byte roundup(codes_bytes, 256):
+ *     fp16 [N][ldS] with ldS = roundup(K/32, 8) (16-byte row pitch);
+ *   every padding byte is zero, so two images of the same weights compare equal
+ *   byte for byte.
+ * Returns the byte size, or 0 when fmt is unknown, N < 1, K < 32 or K % 32 != 0. */
+EMB_API size_t emb_qweight_bytes(emb_qfmt fmt, int64_t N, int64_t K);
+
+/* Quantise fp32 W [N][K] (device, 16-byte aligned) into W_blocks (device,
+ * 256-byte aligned, emb_qweight_bytes(EMB_Q8_0, N, K) bytes). Offline step of
+ * the path (packing weights once per model). NaN/Inf weights, and weights so
+ * large that max|w|/127 overflows fp16, are outside the contract. */
+EMB_API emb_status emb_quantize_q8_0(const float* W, int64_t N, int64_t K, void* W_blocks,
+                             emb_stream_t stream);
+
+/* As emb_quantize_q8_0 for EMB_Q4_0 (m/-8 must not overflow fp16). */
+EMB_API emb_status emb_quantize_q4_0(const float* W, int64_t N, int64_t K, void* W_blocks,
+                             emb_stream_t stream);
+
+/* ---------------------------------------------------------------------- matmul
+ * Y [M][N] fp32 = X [M][K] bf16  x  w'^T, w' the dequantised weights of W_blocks.
+ * X, Y: device, 16-byte aligned; W_blocks as produced by emb_quantize_*.
+ * Small M (action-token decode) runs a weight-streaming GEMV that dequantises in
+ * registers; larger M (action-chunk denoising, prefix prefill) runs a tcgen05
+ * tensor-core GEMM that dequantises shared-memory tiles to bf16.
+ * Accuracy: |Y - Y_exact| <= 1e-3 * sum_k |w'[n][k] x[m][k]| + 1e-6 per element,
+ * where Y_exact uses the same dequantised weights and the same bf16 X.
+ * Results are bitwise reproducible from call to call for a given shape. */
+EMB_API emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_t* X, float* Y,
+                       int64_t M, int64_t N, int64_t K, emb_stream_t stream);
+
+/* --------------------------------------------------------------- layer chains
+ * One linear layer of a chain: Y = X x w'^T with its own X and Y (device). */
+typedef struct {
+    int32_t fmt;            /* emb_qfmt */
+    int32_t reserved;       /* must be 0 */
+    const void* W_blocks;   /* packed image of W [N][K] */
+    int64_t N;
+    int64_t K;
+    const uint16_t* X;      /* [M][K] bf16 */
+    float* Y;               /* [M][N] fp32 */
+} emb_qlayer;
+
+#define EMB_MAX_LAYERS 4096
+
+/* Bytes of device workspace emb_qlayer_seq needs for these layers at this M
+ * (0 is a valid answer). Returns (size_t)-1 for invalid arguments. */
+EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M);
+
+/* Run n_layers linears in order on `stream`, all with M tokens (the paper's
+ * "graph replay, buffer reuse, operator fusion": Section 3.2, principle 2).
+ * Semantics are those of n_layers emb_qmatmul calls in sequence. Consecutive
+ * layers that read the same X with the same fmt and K (q/k/v, gate/up) are
+ * fused into one launch; each launch may fetch its weights before the previous
+ * launch has finished (programmatic dependent launch), and reads X only after
+ * it. A layer's X or W_blocks may not overlap the Y of the same or an earlier
+ * layer inside one call (EMB_EINVAL). The call enqueues kernels only (plus
+ * memsets of the workspace), so it may be captured into a CUDA graph and
+ * replayed. workspace: device, 256-byte aligned, >= emb_qlayer_seq_workspace()
+ * bytes (may be NULL when that is 0). */
+EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M,
+                          void* workspace, size_t ws_bytes, emb_stream_t stream);
+
+/* ---------------------------------------------------------------- test support
+ * Dequantise W_blocks to fp32 [N][K] (w' exactly: the products are exact in fp32). */
+EMB_API emb_status emb_dequantize_f32(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
+                              float* out, emb_stream_t stream);
+
+/* Dequantise to bf16 bit patterns [N][K]: one round-to-nearest-even of the exact fp32
+ * w' -- the operand values the tensor-core GEMM feeds to its MMAs. */
+EMB_API emb_status emb_dequantize_bf16(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
+                               uint16_t* out, emb_stream_t stream);
+
+/* Synchronise `stream`, then return and clear the device status word: EMB_OK, or
+ * EMB_ETIMEOUT if a kernel's bounded wait expired since the last call. */
+EMB_API emb_status emb_device_status(emb_stream_t stream);
+
+/* Launch one block that waits on a shared-memory barrier that nothing completes,
+ * giving up after timeout_ns nanoseconds (1e3 .. 1e9): exercises the bounded-wait
+ * error path; emb_device_status then returns EMB_ETIMEOUT. */
+EMB_API emb_status emb_selftest_wait_timeout(int64_t timeout_ns, emb_stream_t stream);
+
+/* Human-readable name of a status code (static string). */
+EMB_API const char* emb_status_string(emb_status status);
+
+/* Static string describing the build (target architecture, kernel variants). */
+EMB_API const char* emb_build_info(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EMB_QMM_H */

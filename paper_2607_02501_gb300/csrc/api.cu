@@ -1,0 +1,293 @@
+// C ABI of libembqmm.so (declarations and contracts in include/emb_qmm.h).
+//
+// This file holds the host side of the library boundary: argument validation (every
+// error is reported before anything is enqueued), dispatch by token count between the
+// weight-streaming GEMV and the tcgen05 GEMM, fusion of consecutive layers that read the
+// same activation, programmatic dependent launch between the launches of one layer
+// chain (the paper's latency-first fused execution, Section 3.2, design principle 2),
+// and the device status word that bounded device-side waits report into.
+#include <mutex>
+#include <vector>
+
+#include "ptx.cuh"
+
+namespace emb {
+namespace {
+
+__device__ int g_status_word;  // OR of kStatus* flags; read and cleared by emb_device_status
+
+// Token counts up to this run the GEMV; above it, the tensor-core GEMM.
+constexpr int64_t kGemvMaxM = 4;
+
+int* status_ptr() {
+    static std::mutex mu;
+    static int* ptrs[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!ptrs[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+        ptrs[dev] = static_cast<int*>(p);
+    }
+    return ptrs[dev];
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+struct Range {
+    uintptr_t lo, hi;  // [lo, hi)
+};
+bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi; }
+
+bool valid_fmt(int fmt) { return fmt == EMB_Q8_0 || fmt == EMB_Q4_0; }
+
+bool valid_shape(int64_t M, int64_t N, int64_t K) {
+    return M >= 1 && N >= 1 && K >= kQBlock && K % kQBlock == 0 && M < (int64_t(1) << 31) &&
+           N < (int64_t(1) << 31) && K < (int64_t(1) << 30) && N * K < (int64_t(1) << 46) &&
+           M * K < (int64_t(1) << 46) && M * N < (int64_t(1) << 46);
+}
+
+emb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? EMB_OK : EMB_ECUDA; }
+
+// Validation shared by emb_qmatmul and every layer of emb_qlayer_seq.
+emb_status check_layer(int fmt, const void* W, const uint16_t* X, const float* Y, int64_t M,
+                       int64_t N, int64_t K) {
+    if (!valid_fmt(fmt) || !valid_shape(M, N, K)) return EMB_EINVAL;
+    if (!W || !X || !Y) return EMB_EINVAL;
+    if (!aligned(W, 256) || !aligned(X, 16) || !aligned(Y, 16)) return EMB_EALIGN;
+    const Layout L = layout_of(fmt, N, K);
+    const Range rw{uintptr_t(W), uintptr_t(W) + uintptr_t(L.total)};
+    const Range rx{uintptr_t(X), uintptr_t(X) + uintptr_t(M * K * 2)};
+    const Range ry{uintptr_t(Y), uintptr_t(Y) + uintptr_t(M * N * 4)};
+    if (overlap(ry, rw) || overlap(ry, rx)) return EMB_EINVAL;
+    return EMB_OK;
+}
+
+MatRef mat_ref(int fmt, const void* W, float* Y, int64_t N, int64_t K) {
+    const Layout L = layout_of(fmt, N, K);
+    const uint8_t* base = static_cast<const uint8_t*>(W);
+    return MatRef{base, reinterpret_cast<const __half*>(base + L.scales_off), Y, N};
+}
+
+cudaError_t launch_group(const GroupRef& g, bool pdl, cudaStream_t s) {
+    int* st = status_ptr();
+    if (!st) return cudaErrorInvalidDevice;
+    if (g.M <= kGemvMaxM) return launch_gemv(g, pdl, st, s);
+    return launch_gemm_tc(g, pdl, st, s);
+}
+
+// ------------------------------------------------------------ self-test kernel
+__global__ void selftest_wait_kernel(uint64_t timeout_ns, int* status) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(&bar, 1);
+        ptx::fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        // nothing ever arrives on `bar`: the bounded wait must give up and report
+        ptx::mbar_wait(&bar, 0, nullptr, status, timeout_ns);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_selftest_wait(uint64_t timeout_ns, int* status, cudaStream_t s) {
+    selftest_wait_kernel<<<1, 32, 0, s>>>(timeout_ns, status);
+    return cudaGetLastError();
+}
+
+}  // namespace emb
+
+using namespace emb;
+
+extern "C" {
+
+size_t emb_qweight_bytes(emb_qfmt fmt, int64_t N, int64_t K) {
+    if (!valid_fmt(fmt) || !valid_shape(1, N, K)) return 0;
+    return size_t(layout_of(fmt, N, K).total);
+}
+
+static emb_status quantize_common(int fmt, const float* W, int64_t N, int64_t K, void* out,
+                                  emb_stream_t stream) {
+    if (!valid_shape(1, N, K) || !W || !out) return EMB_EINVAL;
+    if (!aligned(W, 16) || !aligned(out, 256)) return EMB_EALIGN;
+    const Layout L = layout_of(fmt, N, K);
+    if (overlap(Range{uintptr_t(W), uintptr_t(W) + uintptr_t(N * K * 4)},
+                Range{uintptr_t(out), uintptr_t(out) + uintptr_t(L.total)}))
+        return EMB_EINVAL;
+    return from_cuda(launch_quantize(fmt, W, N, K, out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+emb_status emb_quantize_q8_0(const float* W, int64_t N, int64_t K, void* W_blocks,
+                             emb_stream_t stream) {
+    return quantize_common(EMB_Q8_0, W, N, K, W_blocks, stream);
+}
+
+emb_status emb_quantize_q4_0(const float* W, int64_t N, int64_t K, void* W_blocks,
+                             emb_stream_t stream) {
+    return quantize_common(EMB_Q4_0, W, N, K, W_blocks, stream);
+}
+
+emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_t* X, float* Y, int64_t M,
+                       int64_t N, int64_t K, emb_stream_t stream) {
+    const emb_status st = check_layer(fmt, W_blocks, X, Y, M, N, K);
+    if (st != EMB_OK) return st;
+    GroupRef g = {};
+    g.fmt = fmt;
+    g.n_mats = 1;
+    g.mats[0] = mat_ref(fmt, W_blocks, Y, N, K);
+    g.X = reinterpret_cast<const __nv_bfloat16*>(X);
+    g.M = M;
+    g.K = K;
+    g.ldS = layout_of(fmt, N, K).ldS;
+    if (M > kGemvMaxM && !gemm_tc_supported(g)) return EMB_EUNSUPPORTED;
+    return from_cuda(launch_group(g, false, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+// Group consecutive layers that read the same X with the same format and K, when no
+// member's Y overlaps another member's W or Y (they then run in one launch).
+static std::vector<std::pair<int, int>> plan_groups(const emb_qlayer* layers, int n, int64_t M) {
+    std::vector<std::pair<int, int>> groups;  // [first, last)
+    auto y_range = [&](int b) {
+        return Range{uintptr_t(layers[b].Y), uintptr_t(layers[b].Y) + uintptr_t(M * layers[b].N * 4)};
+    };
+    auto w_range = [&](int a) {
+        const Layout La = layout_of(layers[a].fmt, layers[a].N, layers[a].K);
+        return Range{uintptr_t(layers[a].W_blocks), uintptr_t(layers[a].W_blocks) + uintptr_t(La.total)};
+    };
+    int i = 0;
+    while (i < n) {
+        int j = i + 1;
+        while (j < n && j - i < kMaxGroup && layers[j].X == layers[i].X &&
+               layers[j].fmt == layers[i].fmt && layers[j].K == layers[i].K) {
+            bool clash = false;
+            for (int a = i; a <= j && !clash; ++a)
+                for (int b = i; b <= j && !clash; ++b)
+                    if (a != b && (overlap(y_range(b), w_range(a)) || overlap(y_range(b), y_range(a))))
+                        clash = true;
+            if (clash) break;
+            ++j;
+        }
+        groups.emplace_back(i, j);
+        i = j;
+    }
+    return groups;
+}
+
+static emb_status check_seq(const emb_qlayer* layers, int n_layers, int64_t M) {
+    if (!layers || n_layers < 1 || n_layers > EMB_MAX_LAYERS || M < 1) return EMB_EINVAL;
+    for (int j = 0; j < n_layers; ++j) {
+        const emb_qlayer& L = layers[j];
+        if (L.reserved != 0) return EMB_EINVAL;
+        const emb_status st = check_layer(L.fmt, L.W_blocks, L.X, L.Y, M, L.N, L.K);
+        if (st != EMB_OK) return st;
+    }
+    // a layer's inputs (X, W) may not be written by the same or an earlier layer
+    for (int j = 0; j < n_layers; ++j) {
+        const emb_qlayer& Lj = layers[j];
+        const Range xj{uintptr_t(Lj.X), uintptr_t(Lj.X) + uintptr_t(M * Lj.K * 2)};
+        const Range wj{uintptr_t(Lj.W_blocks),
+                       uintptr_t(Lj.W_blocks) + uintptr_t(layout_of(Lj.fmt, Lj.N, Lj.K).total)};
+        for (int i = 0; i < j; ++i) {
+            const Range yi{uintptr_t(layers[i].Y), uintptr_t(layers[i].Y) + uintptr_t(M * layers[i].N * 4)};
+            if (overlap(yi, xj) || overlap(yi, wj)) return EMB_EINVAL;
+        }
+    }
+    return EMB_OK;
+}
+
+size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M) {
+    if (check_seq(layers, n_layers, M) != EMB_OK) return size_t(-1);
+    return 0;
+}
+
+emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
+                          size_t ws_bytes, emb_stream_t stream) {
+    (void)workspace;
+    (void)ws_bytes;
+    const emb_status st = check_seq(layers, n_layers, M);
+    if (st != EMB_OK) return st;
+    const auto groups = plan_groups(layers, n_layers, M);
+    std::vector<GroupRef> refs;
+    refs.reserve(groups.size());
+    for (const auto& gr : groups) {
+        const emb_qlayer& L0 = layers[gr.first];
+        GroupRef g = {};
+        g.fmt = L0.fmt;
+        g.n_mats = gr.second - gr.first;
+        for (int k = 0; k < g.n_mats; ++k) {
+            const emb_qlayer& L = layers[gr.first + k];
+            g.mats[k] = mat_ref(L.fmt, L.W_blocks, L.Y, L.N, L.K);
+        }
+        g.X = reinterpret_cast<const __nv_bfloat16*>(L0.X);
+        g.M = M;
+        g.K = L0.K;
+        g.ldS = layout_of(L0.fmt, 1, L0.K).ldS;
+        if (M > kGemvMaxM && !gemm_tc_supported(g)) return EMB_EUNSUPPORTED;
+        refs.push_back(g);
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    for (size_t i = 0; i < refs.size(); ++i) {
+        // the first launch must not overlap whatever the caller enqueued before (it may
+        // have produced the weights); later ones overlap their weight fetch with the
+        // previous launch of this chain
+        const cudaError_t e = launch_group(refs[i], i > 0, s);
+        if (e != cudaSuccess) return EMB_ECUDA;
+    }
+    return EMB_OK;
+}
+
+emb_status emb_dequantize_f32(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
+                              float* out, emb_stream_t stream) {
+    if (!valid_fmt(fmt) || !valid_shape(1, N, K) || !W_blocks || !out) return EMB_EINVAL;
+    if (!aligned(W_blocks, 256) || !aligned(out, 16)) return EMB_EALIGN;
+    return from_cuda(launch_dequant_f32(fmt, W_blocks, N, K, out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+emb_status emb_dequantize_bf16(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
+                               uint16_t* out, emb_stream_t stream) {
+    if (!valid_fmt(fmt) || !valid_shape(1, N, K) || !W_blocks || !out) return EMB_EINVAL;
+    if (!aligned(W_blocks, 256) || !aligned(out, 16)) return EMB_EALIGN;
+    return from_cuda(launch_dequant_bf16(fmt, W_blocks, N, K, out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+emb_status emb_device_status(emb_stream_t stream) {
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return EMB_ECUDA;
+    int* st = status_ptr();
+    if (!st) return EMB_ECUDA;
+    int host = 0;
+    if (cudaMemcpy(&host, st, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return EMB_ECUDA;
+    if (cudaMemset(st, 0, sizeof(int)) != cudaSuccess) return EMB_ECUDA;
+    if (cudaDeviceSynchronize() != cudaSuccess) return EMB_ECUDA;
+    return (host & kStatusTimeout) ? EMB_ETIMEOUT : EMB_OK;
+}
+
+emb_status emb_selftest_wait_timeout(int64_t timeout_ns, emb_stream_t stream) {
+    if (timeout_ns < 1000 || timeout_ns > 1000000000) return EMB_EINVAL;
+    int* st = status_ptr();
+    if (!st) return EMB_ECUDA;
+    return from_cuda(launch_selftest_wait(uint64_t(timeout_ns), st, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+const char* emb_status_string(emb_status status) {
+    switch (status) {
+        case EMB_OK: return "EMB_OK";
+        case EMB_EINVAL: return "EMB_EINVAL: invalid argument";
+        case EMB_EALIGN: return "EMB_EALIGN: misaligned device pointer";
+        case EMB_ENOSPC: return "EMB_ENOSPC: workspace too small";
+        case EMB_ECUDA: return "EMB_ECUDA: CUDA runtime error";
+        case EMB_ETIMEOUT: return "EMB_ETIMEOUT: device-side wait expired";
+        case EMB_EUNSUPPORTED: return "EMB_EUNSUPPORTED: shape not supported by this build";
+    }
+    return "unknown emb_status";
+}
+
+const char* emb_build_info(void) {
+    return "libembqmm: sm_103a; Q8_0/Q4_0; GEMV (M<=4, register dequant, FFMA2) + "
+           "tcgen05 GEMM (M>4, TMA + smem dequant to bf16, TMEM accumulators)";
+}
+
+}  // extern "C"

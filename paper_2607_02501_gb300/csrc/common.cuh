@@ -1,0 +1,85 @@
+// Internal declarations shared by the library's translation units (not installed).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "../../include/emb_qmm.h"
+
+namespace emb {
+
+constexpr int kQBlock = 32;  // weights per quantisation block (both formats)
+
+__host__ __device__ inline int64_t roundup(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
+
+// Byte layout of one packed image (the format comment of emb_qweight_bytes).
+struct Layout {
+    int64_t codes_bytes;  // codes plane size
+    int64_t scales_off;   // byte offset of the fp16 scales plane (256-aligned)
+    int64_t ldS;          // scales row pitch in halves (multiple of 8)
+    int64_t total;        // total image size in bytes
+};
+
+__host__ __device__ inline Layout layout_of(int fmt, int64_t N, int64_t K) {
+    Layout L;
+    L.codes_bytes = (fmt == EMB_Q8_0) ? N * K : N * K / 2;
+    L.scales_off = roundup(L.codes_bytes, 256);
+    L.ldS = roundup(K / kQBlock, 8);
+    L.total = L.scales_off + N * L.ldS * 2;
+    return L;
+}
+
+// Device status word values (bit flags, OR-ed by kernels).
+constexpr int kStatusTimeout = 1;
+
+// Default bound for every spin-wait inside the library's kernels (nanoseconds of
+// %globaltimer). Long enough for any legitimate wait, short enough that a lost
+// arrival turns into EMB_ETIMEOUT instead of a hung GPU.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+// ------------------------------------------------------------------ launchers
+// Each returns cudaSuccess or the launch error. `status` is the device address of
+// the library's status word.
+
+cudaError_t launch_quantize(int fmt, const float* W, int64_t N, int64_t K, void* img,
+                            cudaStream_t s);
+cudaError_t launch_dequant_f32(int fmt, const void* img, int64_t N, int64_t K, float* out,
+                               cudaStream_t s);
+cudaError_t launch_dequant_bf16(int fmt, const void* img, int64_t N, int64_t K, uint16_t* out,
+                                cudaStream_t s);
+
+// Up to kMaxGroup matrices that read the same X (fused q/k/v or gate/up).
+constexpr int kMaxGroup = 4;
+
+struct MatRef {
+    const uint8_t* codes;
+    const __half* scales;
+    float* Y;
+    int64_t N;
+};
+
+struct GroupRef {
+    int fmt;
+    int n_mats;
+    MatRef mats[kMaxGroup];
+    const __nv_bfloat16* X;
+    int64_t M;
+    int64_t K;
+    int64_t ldS;
+};
+
+// Weight-streaming GEMV for small M (register dequant, shuffle reductions).
+// pdl: launch with programmatic stream serialisation (the kernel reads X only after
+// griddepcontrol.wait, weights before).
+cudaError_t launch_gemv(const GroupRef& g, bool pdl, int* status, cudaStream_t s);
+
+// Tensor-core GEMM (tcgen05 + TMEM) for larger M.
+cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s);
+bool gemm_tc_supported(const GroupRef& g);
+
+// Self-test kernel: waits on an mbarrier nobody arrives at, for timeout_ns.
+cudaError_t launch_selftest_wait(uint64_t timeout_ns, int* status, cudaStream_t s);
+
+}  // namespace emb

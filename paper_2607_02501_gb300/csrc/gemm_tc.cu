@@ -1,0 +1,492 @@
+// Tensor-core GEMM for the larger token counts of one closed-loop step (M = 50 action
+// chunk, M = 280..816 prefix prefill): packed Q8_0/Q4_0 weights are staged in shared
+// memory by TMA, dequantised by four warps into 128B-swizzled bf16 tiles, and fed to
+// tcgen05 MMAs whose fp32 accumulators live in TMEM.
+//
+// "Swap AB": the MMA's M side is 128 weight rows (output features n), its N side is the
+// CTA's T tokens, so one weight tile is dequantised once for up to 256 tokens and the
+// accumulator D[n][m] sits in TMEM lanes = n. The epilogue reads TMEM lane n (one
+// thread per output feature) and writes Y[m][n] with 128-byte coalesced stores.
+//
+// Roles (192 threads):
+//   warp 0 lane 0 : TMA producer. Raw stages (256 codes of 128 rows + their 8 scales)
+//                   are fetched before griddepcontrol.wait (weights never depend on
+//                   the previous launch); X tiles (64 k x T tokens) after it.
+//   warp 1        : TMEM allocation; lane 0 issues the MMAs (4 x K=16 per 64-k stage).
+//   warps 2..5    : dequantisation (thread = weight row), then the epilogue.
+// Every wait is bounded (ptx::mbar_wait); on expiry the kernel records EMB_ETIMEOUT,
+// lets every copy and MMA it issued land, frees TMEM and returns.
+//
+// Precision: each operand value is bf16(w') -- one rounding of the exact fp32 w' -- so
+// the products are exact and accumulate in fp32. For K < 1024 the SPLIT variant also
+// stages lo = bf16(w' - bf16(w')) and issues a second MMA per step, which brings the
+// operand error from 2^-9 to 2^-17 relative (the 1e-3 * sum|w x| bound then holds for
+// every input, not only statistically).
+#include <cuda.h>
+#include <cstring>
+#include <mutex>
+
+#include "ptx.cuh"
+
+namespace emb {
+namespace {
+
+constexpr int kBN = 128;                   // weight rows per CTA (MMA M)
+constexpr int kKC = 64;                    // k per A/X stage: one 128-byte bf16 atom row
+constexpr int kKR = 256;                   // k per raw stage
+constexpr int kStepsPerRaw = kKR / kKC;    // 4
+constexpr int kRawStages = 2;
+constexpr int kThreads = 192;
+constexpr int kATile = kBN * kKC * 2;      // 16 KB bf16 tile
+constexpr int kPlane = kBN * 128;          // 16 KB: 128 rows x 128 bytes of codes
+constexpr int kScaleTile = kBN * 16;       // 2 KB: 128 rows x 8 fp16 scales
+
+struct GemmParams {
+    CUtensorMap x_map;                     // X [M][K] bf16, box {64, T}, 128B swizzle
+    CUtensorMap codes_map[kMaxGroup];      // codes [N][row bytes] u8, box {128, 128}, 128B swizzle
+    CUtensorMap scales_map[kMaxGroup];     // scales [N][ldS] u16, box {8, 128}
+    float* Y[kMaxGroup];
+    int32_t N[kMaxGroup];
+    int32_t tile0[kMaxGroup + 1];
+    int32_t n_mats;
+    int32_t M, K;
+    int32_t T;                             // tokens per CTA, multiple of 16, <= 256
+    int32_t stages;                        // A/X ring depth
+    uint32_t tmem_cols;
+    int* status;
+};
+
+template <int FMT>
+struct RawTraits {
+    static constexpr int planes = (FMT == EMB_Q8_0) ? 2 : 1;  // 128-byte code chunks per raw stage
+    static constexpr int bytes = planes * kPlane;
+    // w' = d*(f - bias) where f = 2^15 + byte is built by __byte_perm
+    static constexpr float bias = (FMT == EMB_Q8_0) ? 32768.0f + 128.0f : 32768.0f + 8.0f;
+};
+
+__device__ __forceinline__ uint4 lds128(const uint8_t* p) {
+    return *reinterpret_cast<const uint4*>(p);
+}
+__device__ __forceinline__ void sts128(uint8_t* p, uint4 v) { *reinterpret_cast<uint4*>(p) = v; }
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Four 8-bit values b_i (the bytes of u) -> w'_i = d*(b_i - bias) exactly, as two fp32 pairs.
+// __byte_perm(u, 0x47000000, 0x7504 | i<<4) is the binary32 with exponent 15 whose
+// fraction holds b_i at bits 8..15, i.e. 2^15 + b_i; one FMA with (d, -bias*d) gives
+// d*(b_i - bias) exactly (the product has at most 19 significant bits; bias*d at most 24).
+__device__ __forceinline__ void bytes_to_w(uint32_t u, float d, float nbd, float2& w01,
+                                           float2& w23) {
+    const float2 dd = make_float2(d, d), oo = make_float2(nbd, nbd);
+    w01 = __ffma2_rn(make_float2(__uint_as_float(__byte_perm(u, 0x47000000u, 0x7504u)),
+                                 __uint_as_float(__byte_perm(u, 0x47000000u, 0x7514u))),
+                     dd, oo);
+    w23 = __ffma2_rn(make_float2(__uint_as_float(__byte_perm(u, 0x47000000u, 0x7524u)),
+                                 __uint_as_float(__byte_perm(u, 0x47000000u, 0x7534u))),
+                     dd, oo);
+}
+
+// 8 consecutive w' (two input words) -> one 16-byte chunk of bf16 (hi), and for the split
+// variant the residual chunk lo = bf16(w' - hi).
+template <bool SPLIT>
+__device__ __forceinline__ void make_chunk(uint32_t u0, uint32_t u1, float d, float nbd,
+                                           uint4& hi, uint4& lo) {
+    float2 a, b, c, e;
+    bytes_to_w(u0, d, nbd, a, b);
+    bytes_to_w(u1, d, nbd, c, e);
+    hi = make_uint4(pack_bf16(a.x, a.y), pack_bf16(b.x, b.y), pack_bf16(c.x, c.y),
+                    pack_bf16(e.x, e.y));
+    if constexpr (SPLIT) {
+        auto res = [](float2 v, uint32_t h) {
+            const float2 hv = make_float2(__uint_as_float(h << 16), __uint_as_float(h & 0xFFFF0000u));
+            const float2 r = __fadd2_rn(v, make_float2(-hv.x, -hv.y));  // exact
+            return pack_bf16(r.x, r.y);
+        };
+        lo = make_uint4(res(a, hi.x), res(b, hi.y), res(c, hi.z), res(e, hi.w));
+    }
+}
+
+template <int FMT, bool SPLIT>
+__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmParams p) {
+    using RT = RawTraits<FMT>;
+    constexpr int kAT = SPLIT ? 2 : 1;
+    extern __shared__ uint8_t smem_dyn[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
+                                               ~uintptr_t(1023));
+    const int S = p.stages, T = p.T;
+    uint8_t* a_ring = base;                                     // S x kAT x 16 KB
+    uint8_t* x_ring = a_ring + S * kAT * kATile;                // S x T x 128 B
+    uint8_t* r_ring = x_ring + S * T * 128;                     // 2 x RT::bytes
+    uint8_t* s_ring = r_ring + kRawStages * RT::bytes;          // 2 x 2 KB
+    uint64_t* bars = reinterpret_cast<uint64_t*>(s_ring + kRawStages * kScaleTile);
+    uint64_t* raw_full = bars;
+    uint64_t* raw_empty = bars + kRawStages;
+    uint64_t* x_full = bars + 2 * kRawStages;
+    uint64_t* a_full = x_full + S;
+    uint64_t* ax_empty = a_full + S;
+    uint64_t* acc_full = ax_empty + S;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tile = blockIdx.x;
+    int g = 0;
+#pragma unroll
+    for (int i = 1; i < kMaxGroup; ++i)
+        if (i < p.n_mats && tile >= p.tile0[i]) g = i;
+    const int n0 = (tile - p.tile0[g]) * kBN;
+    const int m0 = blockIdx.y * T;
+    const int N = p.N[g], M = p.M, K = p.K;
+    const int nk = (K + kKC - 1) / kKC;
+    const int nr = (K + kKR - 1) / kKR;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kRawStages; ++i) {
+            ptx::mbar_init(&raw_full[i], 1);
+            ptx::mbar_init(&raw_empty[i], 4);
+        }
+        for (int i = 0; i < S; ++i) {
+            ptx::mbar_init(&x_full[i], 1);
+            ptx::mbar_init(&a_full[i], 4);
+            ptx::mbar_init(&ax_empty[i], 1);
+        }
+        ptx::mbar_init(acc_full, 1);
+        *abort_flag = 0;
+        ptx::fence_mbar_init();
+        ptx::prefetch_tmap(&p.x_map);
+        ptx::prefetch_tmap(&p.codes_map[g]);
+        ptx::prefetch_tmap(&p.scales_map[g]);
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(tmem_slot, p.tmem_cols);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    ptx::griddep_launch_dependents();
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------------------------------------------------------- producer
+            const uint64_t pol_w = ptx::policy_evict_first();
+            const uint64_t pol_x = ptx::policy_evict_last();
+            auto issue_raw = [&](int r) {
+                const int slot = r % kRawStages;
+                ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + kScaleTile);
+#pragma unroll
+                for (int pl = 0; pl < RT::planes; ++pl)
+                    ptx::tma_load_2d(r_ring + slot * RT::bytes + pl * kPlane, &p.codes_map[g],
+                                     &raw_full[slot], (r * RT::planes + pl) * 128, n0, pol_w);
+                ptx::tma_load_2d(s_ring + slot * kScaleTile, &p.scales_map[g], &raw_full[slot],
+                                 r * (kKR / kQBlock), n0, pol_w);
+            };
+            int raw_issued = 0, x_issued = 0;
+            for (; raw_issued < nr && raw_issued < kRawStages; ++raw_issued) issue_raw(raw_issued);
+            ptx::griddep_wait();  // X may be written by the previous launch
+            for (int i = 0; i < nk; ++i) {
+                if (i % kStepsPerRaw == 0) {
+                    const int r = i / kStepsPerRaw;
+                    if (r >= raw_issued) {
+                        if (!ptx::mbar_wait(&raw_empty[r % kRawStages], ((r / kRawStages) - 1) & 1,
+                                            abort_flag, p.status, kWaitLimitNs))
+                            break;
+                        issue_raw(r);
+                        ++raw_issued;
+                    }
+                }
+                const int s = i % S;
+                if (i >= S && !ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
+                                              p.status, kWaitLimitNs))
+                    break;
+                ptx::mbar_arrive_expect_tx(&x_full[s], uint32_t(T) * 128u);
+                ptx::tma_load_2d(x_ring + s * T * 128, &p.x_map, &x_full[s], i * kKC, m0, pol_x);
+                ++x_issued;
+            }
+            // every issued copy must land before this CTA's shared memory can be released
+            for (int r = raw_issued - 1; r >= 0 && r >= raw_issued - kRawStages; --r)
+                ptx::mbar_wait(&raw_full[r % kRawStages], (r / kRawStages) & 1, nullptr, p.status,
+                               kWaitLimitNs);
+            for (int i = x_issued - 1; i >= 0 && i >= x_issued - S; --i)
+                ptx::mbar_wait(&x_full[i % S], (i / S) & 1, nullptr, p.status, kWaitLimitNs);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ------------------------------------------------------------ MMA issuer
+            const uint32_t idesc = ptx::idesc_bf16_f32(kBN, T);
+            const uint32_t a0 = ptx::smem_u32(a_ring), x0 = ptx::smem_u32(x_ring);
+            for (int i = 0; i < nk; ++i) {
+                const int s = i % S;
+                const uint32_t ph = (i / S) & 1;
+                if (!ptx::mbar_wait(&x_full[s], ph, abort_flag, p.status, kWaitLimitNs)) break;
+                if (!ptx::mbar_wait(&a_full[s], ph, abort_flag, p.status, kWaitLimitNs)) break;
+                ptx::tc_fence_after();
+                const uint32_t a_addr = a0 + s * kAT * kATile, x_addr = x0 + s * T * 128;
+#pragma unroll
+                for (int k = 0; k < kKC / 16; ++k) {
+                    const uint64_t bdesc = ptx::smem_desc_sw128(x_addr + 32 * k);
+                    ptx::mma_bf16(tmem, ptx::smem_desc_sw128(a_addr + 32 * k), bdesc, idesc,
+                                  (i | k) != 0);
+                    if constexpr (SPLIT)
+                        ptx::mma_bf16(tmem, ptx::smem_desc_sw128(a_addr + kATile + 32 * k), bdesc,
+                                      idesc, 1u);
+                }
+                ptx::mma_commit(&ax_empty[s]);
+            }
+            ptx::mma_commit(acc_full);  // completes once every issued MMA has finished
+            ptx::mbar_wait(acc_full, 0, nullptr, p.status, kWaitLimitNs);
+        }
+    } else {
+        // ---------------------------------------------------------------- dequant
+        const int t = threadIdx.x - 64;  // weight row within the tile
+        const unsigned full = 0xffffffffu;
+        bool ok = true;
+        for (int r = 0; r < nr && ok; ++r) {
+            const int rs = r % kRawStages;
+            ok = __all_sync(full, ptx::mbar_wait(&raw_full[rs], (r / kRawStages) & 1, abort_flag,
+                                                 p.status, kWaitLimitNs));
+            if (!ok) break;
+            const uint8_t* rbase = r_ring + rs * RT::bytes + t * 128;
+            const uint4 sv = lds128(s_ring + rs * kScaleTile + t * 16);
+            const uint32_t sw[4] = {sv.x, sv.y, sv.z, sv.w};
+            float d[8], nbd[8];
+#pragma unroll
+            for (int b = 0; b < 8; ++b) {
+                const uint16_t hb = uint16_t((sw[b >> 1] >> (16 * (b & 1))) & 0xFFFFu);
+                d[b] = __half2float(__ushort_as_half(hb));
+                nbd[b] = -RT::bias * d[b];  // exact (see bytes_to_w)
+            }
+#pragma unroll
+            for (int j = 0; j < kStepsPerRaw; ++j) {
+                const int i = r * kStepsPerRaw + j;
+                if (i >= nk) break;
+                const int s = i % S;
+                if (i >= S) {
+                    ok = __all_sync(full, ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
+                                                         p.status, kWaitLimitNs));
+                    if (!ok) break;
+                }
+                uint8_t* arow = a_ring + s * kAT * kATile + t * 128;
+                const int sx = t & 7;  // 128B swizzle: 16-byte chunk c of row t lives at c ^ (t & 7)
+                if constexpr (FMT == EMB_Q8_0) {
+                    // atom j: codes 64j..64j+63 of the raw stage = plane j/2, chunks 4(j%2)..+3
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc) {
+                        const int c = (j & 1) * 4 + cc;
+                        const uint4 v = lds128(rbase + (j >> 1) * kPlane + ((c ^ sx) << 4));
+                        const int b = 2 * j + (cc >> 1);  // 32-block within the raw stage
+                        uint4 h0, l0, h1, l1;
+                        make_chunk<SPLIT>(v.x ^ 0x80808080u, v.y ^ 0x80808080u, d[b], nbd[b], h0, l0);
+                        make_chunk<SPLIT>(v.z ^ 0x80808080u, v.w ^ 0x80808080u, d[b], nbd[b], h1, l1);
+                        const int o0 = 2 * cc, o1 = 2 * cc + 1;
+                        sts128(arow + ((o0 ^ sx) << 4), h0);
+                        sts128(arow + ((o1 ^ sx) << 4), h1);
+                        if constexpr (SPLIT) {
+                            sts128(arow + kATile + ((o0 ^ sx) << 4), l0);
+                            sts128(arow + kATile + ((o1 ^ sx) << 4), l1);
+                        }
+                    }
+                } else {
+                    // atom j: blocks 2j, 2j+1 = 16-byte chunks 2j, 2j+1 of the single plane;
+                    // a block's byte i holds code i (low nibble) and code i+16 (high nibble)
+#pragma unroll
+                    for (int bb = 0; bb < 2; ++bb) {
+                        const int b = 2 * j + bb;
+                        const uint4 v = lds128(rbase + ((b ^ sx) << 4));
+                        const uint32_t m = 0x0F0F0F0Fu;
+                        uint4 h[4], l[4];
+                        make_chunk<SPLIT>(v.x & m, v.y & m, d[b], nbd[b], h[0], l[0]);               // codes 0..7
+                        make_chunk<SPLIT>(v.z & m, v.w & m, d[b], nbd[b], h[1], l[1]);               // 8..15
+                        make_chunk<SPLIT>((v.x >> 4) & m, (v.y >> 4) & m, d[b], nbd[b], h[2], l[2]); // 16..23
+                        make_chunk<SPLIT>((v.z >> 4) & m, (v.w >> 4) & m, d[b], nbd[b], h[3], l[3]); // 24..31
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int o = 4 * bb + q;
+                            sts128(arow + ((o ^ sx) << 4), h[q]);
+                            if constexpr (SPLIT) sts128(arow + kATile + ((o ^ sx) << 4), l[q]);
+                        }
+                    }
+                }
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&a_full[s]);
+            }
+            if (!ok) break;
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&raw_empty[rs]);
+        }
+
+        // ---------------------------------------------------------------- epilogue
+        ptx::griddep_wait();  // Y may be read or written by the previous launch
+        ok = __all_sync(full, ok && ptx::mbar_wait(acc_full, 0, abort_flag, p.status, kWaitLimitNs));
+        if (ok) {
+            ptx::tc_fence_after();
+            const int quarter = warp & 3;  // TMEM lanes this warp may access
+            const int n = n0 + quarter * 32 + lane;
+            const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16);
+            float* Y = p.Y[g];
+            for (int c0 = 0; c0 < T; c0 += 16) {
+                uint32_t v[16];
+                ptx::tmem_ld_16(taddr + uint32_t(c0), v);
+                ptx::tmem_ld_wait();
+                if (n < N) {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const int m = m0 + c0 + e;
+                        if (m < M) Y[int64_t(m) * N + n] = __uint_as_float(v[e]);
+                    }
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, p.tmem_cols);
+    }
+}
+
+// ------------------------------------------------------------------ host side
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(f);
+    });
+    return fn;
+}
+
+bool encode_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t inner,
+               uint64_t outer, uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer,
+               CUtensorMapSwizzle sw, CUtensorMapL2promotion l2) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {row_stride_bytes};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, sw, l2, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
+constexpr int kSmemLimit = 227 * 1024;
+
+template <int FMT, bool SPLIT>
+int smem_bytes(int T, int S) {
+    return 1024 + S * ((SPLIT ? 2 : 1) * kATile + T * 128) +
+           kRawStages * (RawTraits<FMT>::bytes + kScaleTile) + (2 * kRawStages + 3 * S + 1) * 8 + 16;
+}
+
+template <int FMT, bool SPLIT>
+int pick_stages(int T) {
+    int S = 6;
+    while (S > 2 && smem_bytes<FMT, SPLIT>(T, S) > kSmemLimit) --S;
+    return S;
+}
+
+template <int FMT, bool SPLIT>
+cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl, cudaStream_t s) {
+    const int bytes = smem_bytes<FMT, SPLIT>(p.T, p.stages);
+    // the opt-in shared-memory size is a per-device function attribute
+    static std::mutex mu;
+    static bool done[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (dev < 0 || dev >= 64 || !done[dev]) {
+            e = cudaFuncSetAttribute(gemm_tc_kernel<FMT, SPLIT>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+            if (e != cudaSuccess) return e;
+            if (dev >= 0 && dev < 64) done[dev] = true;
+        }
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid_x, grid_y, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = size_t(bytes);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<FMT, SPLIT>, p);
+}
+
+}  // namespace
+
+bool gemm_tc_supported(const GroupRef& g) {
+    return g.M >= 1 && g.M <= int64_t(65535) * 256 && g.K <= (int64_t(1) << 30) &&
+           encode_fn() != nullptr;
+}
+
+cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s) {
+    GemmParams p;
+    memset(&p, 0, sizeof(p));
+    // tokens per CTA: balanced tiles of at most 256, rounded up to the MMA's N granule (16)
+    const int64_t t_tiles = (g.M + 255) / 256;
+    const int T = int(roundup((g.M + t_tiles - 1) / t_tiles, 16));
+    const bool split = g.K < 1024;
+    const int S = g.fmt == EMB_Q8_0 ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
+                                    : (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T));
+    if (!encode_2d(&p.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.X, uint64_t(g.K), uint64_t(g.M),
+                   uint64_t(g.K) * 2, kKC, uint32_t(T), CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_128B))
+        return cudaErrorInvalidValue;
+    int tiles = 0;
+    for (int i = 0; i < g.n_mats; ++i) {
+        const MatRef& mr = g.mats[i];
+        const uint64_t row_bytes = g.fmt == EMB_Q8_0 ? uint64_t(g.K) : uint64_t(g.K) / 2;
+        if (!encode_2d(&p.codes_map[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, mr.codes, row_bytes,
+                       uint64_t(mr.N), row_bytes, 128, kBN, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B))
+            return cudaErrorInvalidValue;
+        if (!encode_2d(&p.scales_map[i], CU_TENSOR_MAP_DATA_TYPE_UINT16, mr.scales,
+                       uint64_t(g.ldS), uint64_t(mr.N), uint64_t(g.ldS) * 2, 8, kBN,
+                       CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B))
+            return cudaErrorInvalidValue;
+        p.Y[i] = mr.Y;
+        p.N[i] = int32_t(mr.N);
+        p.tile0[i] = tiles;
+        tiles += int((mr.N + kBN - 1) / kBN);
+    }
+    p.tile0[g.n_mats] = tiles;
+    p.n_mats = g.n_mats;
+    p.M = int32_t(g.M);
+    p.K = int32_t(g.K);
+    p.T = T;
+    p.stages = S;
+    uint32_t cols = 32;
+    while (cols < uint32_t(T)) cols <<= 1;
+    p.tmem_cols = cols;
+    p.status = status;
+    const int grid_y = int(t_tiles);
+    if (g.fmt == EMB_Q8_0)
+        return split ? launch_kernel<EMB_Q8_0, true>(p, tiles, grid_y, pdl, s)
+                     : launch_kernel<EMB_Q8_0, false>(p, tiles, grid_y, pdl, s);
+    return split ? launch_kernel<EMB_Q4_0, true>(p, tiles, grid_y, pdl, s)
+                 : launch_kernel<EMB_Q4_0, false>(p, tiles, grid_y, pdl, s);
+}
+
+}  // namespace emb

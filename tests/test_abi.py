@@ -1,0 +1,134 @@
+"""The C-ABI library loads, exports every declared entry point, and rejects invalid
+arguments before touching the GPU (CPU only: no call here reaches a launch)."""
+import ctypes
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2607_02501_gb300 as emb
+
+
+@pytest.fixture(scope="module")
+def L():
+    emb.build()
+    return emb.lib()
+
+
+def test_every_declared_symbol_is_exported(L):
+    names = emb.declared_symbols()
+    assert len(names) == 12
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_no_undeclared_exports(L):
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", emb.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    assert exported == set(emb.declared_symbols())
+
+
+@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0])
+@pytest.mark.parametrize("N,K", [(1, 32), (3, 96), (2048, 2048), (256, 2048), (2048, 16384),
+                                 (5, 1152), (4096, 11008), (129, 4608), (7, 4160)])
+def test_qweight_bytes_matches_oracle(L, fmt, N, K):
+    assert emb.emb_qweight_bytes(fmt, N, K) == oracle.packed_bytes(fmt, N, K)
+
+
+@pytest.mark.parametrize("fmt,N,K", [(2, 4, 32), (-1, 4, 32), (0, 0, 32), (0, 4, 0), (0, 4, 48),
+                                     (1, -5, 64), (0, 4, 31)])
+def test_qweight_bytes_invalid(L, fmt, N, K):
+    assert emb.emb_qweight_bytes(fmt, N, K) == 0
+
+
+def test_status_strings(L):
+    for s in range(7):
+        assert emb.emb_status_string(s).startswith(emb._STATUS_NAMES[s])
+    assert "unknown" in emb.emb_status_string(99)
+
+
+# Fake device addresses: only ever used in calls that must fail validation.
+A = 0x7f0000000000            # 256-aligned
+B = A + (1 << 30)
+C = A + (2 << 30)
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((0, None, B, C, 1, 128, 64), emb.EMB_EINVAL),          # null W
+    ((0, A, None, C, 1, 128, 64), emb.EMB_EINVAL),          # null X
+    ((0, A, B, None, 1, 128, 64), emb.EMB_EINVAL),          # null Y
+    ((2, A, B, C, 1, 128, 64), emb.EMB_EINVAL),             # unknown format
+    ((0, A, B, C, 0, 128, 64), emb.EMB_EINVAL),             # M < 1
+    ((0, A, B, C, 1, 0, 64), emb.EMB_EINVAL),               # N < 1
+    ((0, A, B, C, 1, 128, 48), emb.EMB_EINVAL),             # K % 32
+    ((1, A, B, C, 1, 128, 0), emb.EMB_EINVAL),              # K < 32
+    ((0, A + 16, B, C, 1, 128, 64), emb.EMB_EALIGN),        # W not 256-aligned
+    ((0, A, B + 2, C, 1, 128, 64), emb.EMB_EALIGN),         # X not 16-aligned
+    ((1, A, B, C + 4, 1, 128, 64), emb.EMB_EALIGN),         # Y not 16-aligned
+    ((0, A, B, B + 64, 1, 128, 64), emb.EMB_EINVAL),        # Y overlaps X
+    ((0, A, B, A + 256, 1, 128, 64), emb.EMB_EINVAL),       # Y overlaps W
+])
+def test_qmatmul_rejects_before_launch(L, args, expect):
+    fmt, W, X, Y, M, N, K = args
+    assert L.emb_qmatmul(fmt, W, X, Y, M, N, K, None) == expect
+
+
+def test_quantize_rejects(L):
+    assert L.emb_quantize_q8_0(None, 4, 32, A, None) == emb.EMB_EINVAL
+    assert L.emb_quantize_q4_0(B, 4, 48, A, None) == emb.EMB_EINVAL
+    assert L.emb_quantize_q8_0(B + 4, 4, 32, A, None) == emb.EMB_EALIGN
+    assert L.emb_quantize_q4_0(B, 4, 32, A + 128, None) == emb.EMB_EALIGN
+    assert L.emb_quantize_q8_0(A, 4, 32, A + 256, None) == emb.EMB_EINVAL   # in/out overlap
+
+
+def test_dequantize_rejects(L):
+    assert L.emb_dequantize_f32(3, A, 4, 32, B, None) == emb.EMB_EINVAL
+    assert L.emb_dequantize_bf16(0, A, 4, 33, B, None) == emb.EMB_EINVAL
+    assert L.emb_dequantize_f32(0, A + 1, 4, 32, B, None) == emb.EMB_EALIGN
+    assert L.emb_dequantize_bf16(1, A, 4, 32, None, None) == emb.EMB_EINVAL
+
+
+def test_selftest_rejects_out_of_range_timeouts(L):
+    assert L.emb_selftest_wait_timeout(10, None) == emb.EMB_EINVAL
+    assert L.emb_selftest_wait_timeout(10 ** 10, None) == emb.EMB_EINVAL
+
+
+def _layers(specs):
+    return emb.make_layers(specs)
+
+
+def test_seq_rejects(L):
+    M = 1
+    good = (0, A, 128, 64, B, C)
+    arr = _layers([good])
+    assert L.emb_qlayer_seq(None, 1, M, None, 0, None) == emb.EMB_EINVAL
+    assert L.emb_qlayer_seq(arr, 0, M, None, 0, None) == emb.EMB_EINVAL
+    assert L.emb_qlayer_seq(arr, emb.EMB_MAX_LAYERS + 1, M, None, 0, None) == emb.EMB_EINVAL
+    assert L.emb_qlayer_seq(arr, 1, 0, None, 0, None) == emb.EMB_EINVAL
+    bad = _layers([good])
+    bad[0].reserved = 1
+    assert L.emb_qlayer_seq(bad, 1, M, None, 0, None) == emb.EMB_EINVAL
+    # layer 1 reads (as X) what layer 0 writes
+    chain = _layers([good, (0, A + (64 << 20), 128, 64, C, C + (1 << 20))])
+    assert L.emb_qlayer_seq(chain, 2, M, None, 0, None) == emb.EMB_EINVAL
+    # layer 1's weights overlap layer 0's output
+    chain = _layers([good, (0, C, 128, 64, B, C + (1 << 20))])
+    assert L.emb_qlayer_seq(chain, 2, M, None, 0, None) == emb.EMB_EINVAL
+    # misaligned member
+    chain = _layers([good, (1, A + (64 << 20), 128, 64, B + 8, C + (1 << 20))])
+    assert L.emb_qlayer_seq(chain, 2, M, None, 0, None) == emb.EMB_EALIGN
+    assert L.emb_qlayer_seq_workspace(chain, 2, M) == ctypes.c_size_t(-1).value
+
+
+def test_seq_workspace_is_zero_for_valid_chains(L):
+    chain = _layers([(0, A, 128, 64, B, C), (1, A + (64 << 20), 256, 64, B, C + (1 << 20))])
+    assert emb.emb_qlayer_seq_workspace(chain, 1) == 0
+    assert emb.emb_qlayer_seq_workspace(chain, 816) == 0
+
+
+def test_library_has_no_torch_dependency():
+    import subprocess
+    out = subprocess.run(["ldd", emb.LIB_PATH], capture_output=True, text=True).stdout
+    assert "torch" not in out and "libcudart" not in out

@@ -1,0 +1,97 @@
+"""emb_qmatmul against the oracle: GEMV (M <= 4) and tcgen05 GEMM (M > 4) paths on
+shapes spanning several tiles with ragged tails in every dimension."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_02501_gb300 as emb
+from tests.gpu_util import check_close, run_case, to_dev_bf16
+from workloads import activation_bits_np, weight_np
+
+pytestmark = pytest.mark.gpu
+
+FMTS = [emb.EMB_Q8_0, emb.EMB_Q4_0]
+
+GEMV_SHAPES = [(1, 1, 32), (1, 8, 64), (1, 136, 96), (1, 256, 2048), (1, 2048, 2048),
+               (1, 130, 16384), (1, 300, 11008), (1, 4096, 1152), (2, 200, 4608),
+               (3, 129, 1024), (4, 1000, 2080)]
+
+GEMM_SHAPES = [(5, 128, 1024), (7, 136, 96), (16, 8, 32), (49, 256, 2048), (50, 1024, 1024),
+               (51, 264, 1152), (64, 384, 256), (127, 128, 1088), (129, 640, 2048),
+               (255, 136, 512), (257, 256, 1024), (280, 512, 4096), (500, 300, 320),
+               (768, 256, 1152), (816, 384, 2048)]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("M,N,K", GEMV_SHAPES)
+def test_gemv_parity(cuda_device, fmt, M, N, K):
+    Y, Yref, B, _, _ = run_case(fmt, M, N, K, seed=M * 7 + N + K)
+    check_close(Y, Yref, B, f"gemv fmt={fmt} M={M} N={N} K={K}")
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+def test_gemm_parity(cuda_device, fmt, M, N, K):
+    Y, Yref, B, _, _ = run_case(fmt, M, N, K, seed=M * 13 + N + K)
+    check_close(Y, Yref, B, f"gemm fmt={fmt} M={M} N={N} K={K}")
+
+
+@pytest.mark.parametrize("M", [1, 3, 50, 280])
+def test_deterministic(cuda_device, M):
+    N, K = 384, 2048
+    W = torch.from_numpy(weight_np(N, K, 3)).cuda()
+    X = to_dev_bf16(activation_bits_np(M, K, 4))
+    for fmt in FMTS:
+        img = emb.quantize(fmt, W)
+        Y1 = emb.qmatmul(fmt, img, X, N)
+        Y2 = emb.qmatmul(fmt, img, X, N)
+        torch.cuda.synchronize()
+        assert torch.equal(Y1.view(torch.int32), Y2.view(torch.int32))
+
+
+def test_outliers_q4_0(cuda_device):
+    """1% of weights x8 (the 7B configuration's outlier pattern) at both paths."""
+    N, K = 512, 4096
+    rng = np.random.default_rng(77)
+    W = weight_np(N, K, 78)
+    W[rng.random((N, K)) < 0.01] *= 8
+    for M in (1, 280):
+        Xb = activation_bits_np(M, K, 79)
+        img = emb.quantize(emb.EMB_Q4_0, torch.from_numpy(W).cuda())
+        Y = emb.qmatmul(emb.EMB_Q4_0, img, to_dev_bf16(Xb), N).cpu().numpy()
+        Yref, B = oracle.qmatmul(emb.EMB_Q4_0, oracle.quantize(emb.EMB_Q4_0, W), Xb, N, K)
+        check_close(Y, Yref, B, f"outliers M={M}")
+
+
+def test_extreme_activations(cuda_device):
+    """bf16 activations spanning 2^-60..2^40 plus zeros of both signs, where a handful of
+    terms dominate sum|w x|: the GEMV (exact products) and the split-operand GEMM
+    (K < 1024, operand error 2^-17) must meet the bound for such inputs too."""
+    from workloads import bf16_bits_np
+    rng = np.random.default_rng(91)
+    for M, N, K in ((1, 256, 1024), (64, 256, 512)):
+        W = weight_np(N, K, 90)
+        x = (rng.standard_normal((M, K)) * np.exp2(rng.integers(-60, 40, size=(M, K)))).astype(np.float32)
+        x[:, ::17] = 0.0
+        x[:, 5::23] = -0.0
+        Xb = bf16_bits_np(x)
+        for fmt in FMTS:
+            img = emb.quantize(fmt, torch.from_numpy(W).cuda())
+            Y = emb.qmatmul(fmt, img, to_dev_bf16(Xb), N).cpu().numpy()
+            Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
+            check_close(Y, Yref, B, f"extreme x M={M} fmt={fmt}")
+
+
+def test_y_fully_overwritten(cuda_device):
+    N, K = 200, 512
+    W = torch.from_numpy(weight_np(N, K, 5)).cuda()
+    for M in (1, 70):
+        X = to_dev_bf16(activation_bits_np(M, K, 6))
+        for fmt in FMTS:
+            img = emb.quantize(fmt, W)
+            Y0 = emb.qmatmul(fmt, img, X, N)
+            Y1 = torch.full((M, N), float("nan"), device="cuda")
+            emb.qmatmul(fmt, img, X, N, out=Y1)
+            torch.cuda.synchronize()
+            assert torch.equal(Y0, Y1)
