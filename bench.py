@@ -325,6 +325,13 @@ def run_reference(args):
     return 0
 
 
+def truncate(w: wl.Workload, layers: int) -> wl.Workload:
+    import dataclasses
+    layers = max(1, min(layers, w.layers))
+    per = len(w.groups) // w.layers
+    return dataclasses.replace(w, layers=layers, groups=tuple(w.groups[:per * layers]))
+
+
 def metric_name(ws) -> str:
     return "qmatmul µs & HBM GB/s (M=1) / TFLOP/s (M≥50), as fraction of roofline"
 
@@ -350,6 +357,8 @@ def run_ours(args):
     dist = init_dist(world, "nccl")
     emb.lib()
     ws = WORKLOADS[args.workload]()
+    if args.layers:
+        ws = [truncate(w, args.layers) for w in ws]
     chains = []
     for w in ws:
         specs, xs, ys = build_chain(w, dev)
@@ -503,6 +512,9 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="gemma2b_decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run only the first L layers (small cases for ncu captures; "
+                         "a number taken this way is not the workload's bench value)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

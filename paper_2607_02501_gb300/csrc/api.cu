@@ -6,6 +6,7 @@
 // same activation, programmatic dependent launch between the launches of one layer
 // chain (the paper's latency-first fused execution, Section 3.2, design principle 2),
 // and the device status word that bounded device-side waits report into.
+#include <algorithm>
 #include <mutex>
 #include <vector>
 

@@ -15,7 +15,9 @@
 //     programmatic dependent launch a layer's weight stream starts while the previous
 //     layer is still finishing; X is read and Y written only after the wait.
 // Up to kMaxGroup matrices that read the same X (q/k/v or gate/up) share one launch.
-#include "common.cuh"
+#include <mutex>
+
+#include "ptx.cuh"
 
 namespace emb {
 namespace {
@@ -228,20 +230,21 @@ template <int FMT, int R>
 cudaError_t dispatch_nt(const GemvParams& p, int grid_x, int M, int NT, bool pdl, cudaStream_t s) {
     if (NT == 256) return dispatch_mt<FMT, R, 256>(p, grid_x, M, pdl, s);
     if (NT == 128) return dispatch_mt<FMT, R, 128>(p, grid_x, M, pdl, s);
-    return dispatch_mt<FMT, R, 64>(p, grid_x, M, pdl, s);
+    if (NT == 64) return dispatch_mt<FMT, R, 64>(p, grid_x, M, pdl, s);
+    return dispatch_mt<FMT, R, 32>(p, grid_x, M, pdl, s);
 }
 
-// Threads per CTA: the largest of 256/128/64 whose idle lanes in the last K sweep
-// stay under 1/8 of the work, else the one with the least idle lanes.
-int pick_threads(int U) {
-    const int cand[3] = {256, 128, 64};
-    int best = 64, best_waste = 1 << 30;
-    for (int nt : cand) {
-        const int waste = (U + nt - 1) / nt * nt - U;
-        if (waste * 8 <= U) return nt;
-        if (waste < best_waste) { best_waste = waste; best = nt; }
-    }
-    return best;
+// Threads per CTA (they split K): about 8 (Q8_0) or 4 (Q4_0) 16-byte units per thread
+// and row, 32..128 threads, which amortises the per-thread prologue and reduction on large
+// matrices (measured on GB300 at M=1, Q8_0 K=2048: 32 threads 5.6 TB/s, 128 threads
+// 4.6 TB/s). Small matrices are latency-bound instead: there the count grows (up to one
+// unit per thread, 256 threads) until about 152K threads put every byte in flight at once.
+int pick_threads(int U, int fmt, int64_t tiles) {
+    const int target = (fmt == EMB_Q8_0) ? U / 8 : U / 4;
+    int nt = 32;
+    while (nt < 128 && nt < target) nt *= 2;
+    while (nt < 256 && nt < U && tiles * nt < int64_t(152) * 1024) nt *= 2;
+    return nt;
 }
 
 }  // namespace
@@ -269,7 +272,7 @@ cudaError_t launch_gemv(const GroupRef& g, bool pdl, int* /*status*/, cudaStream
     p.ldS = int32_t(g.ldS);
     p.U = U;
     p.X = g.X;
-    const int NT = pick_threads(U);
+    const int NT = pick_threads(U, g.fmt, tiles);
     const int M = int(g.M);
     if (g.fmt == EMB_Q8_0)
         return R == 4 ? dispatch_nt<EMB_Q8_0, 4>(p, tiles, M, NT, pdl, s)
