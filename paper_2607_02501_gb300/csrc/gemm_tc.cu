@@ -8,12 +8,15 @@
 // accumulator D[n][m] sits in TMEM lanes = n. The epilogue reads TMEM lane n (one
 // thread per output feature) and writes Y[m][n] with 128-byte coalesced stores.
 //
-// Roles (192 threads):
+// Roles (320 threads):
 //   warp 0 lane 0 : TMA producer. Raw stages (256 codes of 128 rows + their 8 scales)
 //                   are fetched before griddepcontrol.wait (weights never depend on
 //                   the previous launch); X tiles (64 k x T tokens) after it.
 //   warp 1        : TMEM allocation; lane 0 issues the MMAs (4 x K=16 per 64-k stage).
-//   warps 2..5    : dequantisation (thread = weight row), then the epilogue.
+//   warps 2..9    : dequantisation (two threads per weight row), then the epilogue.
+// Grid: x = token tile (fastest: CTAs sharing a weight tile run together), y = weight-row
+// tile, z = K split. With z > 1 the splits of one output tile form a thread-block cluster
+// and are summed in a fixed order through distributed shared memory (deterministic).
 // Every wait is bounded (ptx::mbar_wait); on expiry the kernel records EMB_ETIMEOUT,
 // lets every copy and MMA it issued land, frees TMEM and returns.
 //
@@ -36,7 +39,8 @@ constexpr int kKC = 64;                    // k per A/X stage: one 128-byte bf16
 constexpr int kKR = 256;                   // k per raw stage
 constexpr int kStepsPerRaw = kKR / kKC;    // 4
 constexpr int kRawStages = 2;
-constexpr int kThreads = 192;
+constexpr int kDeqWarps = 8;               // dequantisation (then epilogue) warps
+constexpr int kThreads = 64 + 32 * kDeqWarps;
 constexpr int kATile = kBN * kKC * 2;      // 16 KB bf16 tile
 constexpr int kPlane = kBN * 128;          // 16 KB: 128 rows x 128 bytes of codes
 constexpr int kScaleTile = kBN * 16;       // 2 KB: 128 rows x 8 fp16 scales
@@ -51,6 +55,7 @@ struct GemmParams {
     int32_t n_mats;
     int32_t M, K;
     int32_t T;                             // tokens per CTA, multiple of 16, <= 256
+    int32_t splits;                        // K splits (cluster size along z)
     int32_t stages;                        // A/X ring depth
     uint32_t tmem_cols;
     int* status;
@@ -130,27 +135,35 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint64_t* acc_full = ax_empty + S;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    // split-K partial tile [T][128] fp32 (token-major): reuses the A/X rings once every
+    // MMA has completed
+    float* part = reinterpret_cast<float*>(a_ring);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile = blockIdx.x;
+    const int tile = blockIdx.y;
     int g = 0;
 #pragma unroll
     for (int i = 1; i < kMaxGroup; ++i)
         if (i < p.n_mats && tile >= p.tile0[i]) g = i;
     const int n0 = (tile - p.tile0[g]) * kBN;
-    const int m0 = blockIdx.y * T;
+    const int m0 = blockIdx.x * T;
     const int N = p.N[g], M = p.M, K = p.K;
-    const int nk = (K + kKC - 1) / kKC;
-    const int nr = (K + kKR - 1) / kKR;
+    // this CTA's K range: split-K over raw stages of 256
+    const int splits = gridDim.z, split = blockIdx.z;
+    const int nr_all = (K + kKR - 1) / kKR, nk_all = (K + kKC - 1) / kKC;
+    const int rs0 = split * nr_all / splits, rs1 = (split + 1) * nr_all / splits;
+    const int nr = rs1 - rs0;
+    const int ks0 = rs0 * kStepsPerRaw;
+    const int nk = min(rs1 * kStepsPerRaw, nk_all) - ks0;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kRawStages; ++i) {
             ptx::mbar_init(&raw_full[i], 1);
-            ptx::mbar_init(&raw_empty[i], 4);
+            ptx::mbar_init(&raw_empty[i], kDeqWarps);
         }
         for (int i = 0; i < S; ++i) {
             ptx::mbar_init(&x_full[i], 1);
-            ptx::mbar_init(&a_full[i], 4);
+            ptx::mbar_init(&a_full[i], kDeqWarps);
             ptx::mbar_init(&ax_empty[i], 1);
         }
         ptx::mbar_init(acc_full, 1);
@@ -177,13 +190,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint64_t pol_x = ptx::policy_evict_last();
             auto issue_raw = [&](int r) {
                 const int slot = r % kRawStages;
+                const int rg = rs0 + r;  // raw stage index within the whole row
                 ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + kScaleTile);
 #pragma unroll
                 for (int pl = 0; pl < RT::planes; ++pl)
                     ptx::tma_load_2d(r_ring + slot * RT::bytes + pl * kPlane, &p.codes_map[g],
-                                     &raw_full[slot], (r * RT::planes + pl) * 128, n0, pol_w);
+                                     &raw_full[slot], (rg * RT::planes + pl) * 128, n0, pol_w);
                 ptx::tma_load_2d(s_ring + slot * kScaleTile, &p.scales_map[g], &raw_full[slot],
-                                 r * (kKR / kQBlock), n0, pol_w);
+                                 rg * (kKR / kQBlock), n0, pol_w);
             };
             int raw_issued = 0, x_issued = 0;
             for (; raw_issued < nr && raw_issued < kRawStages; ++raw_issued) issue_raw(raw_issued);
@@ -204,7 +218,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                                               p.status, kWaitLimitNs))
                     break;
                 ptx::mbar_arrive_expect_tx(&x_full[s], uint32_t(T) * 128u);
-                ptx::tma_load_2d(x_ring + s * T * 128, &p.x_map, &x_full[s], i * kKC, m0, pol_x);
+                ptx::tma_load_2d(x_ring + s * T * 128, &p.x_map, &x_full[s], (ks0 + i) * kKC, m0,
+                                 pol_x);
                 ++x_issued;
             }
             // every issued copy must land before this CTA's shared memory can be released
@@ -242,7 +257,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
     } else {
         // ---------------------------------------------------------------- dequant
-        const int t = threadIdx.x - 64;  // weight row within the tile
+        // two threads per weight row: thread (row t, half h) writes 4 of the 8 16-byte
+        // chunks of each 64-k atom row (the chunks of 32-block 2j+h of atom j)
+        const int u = threadIdx.x - 64;
+        const int t = u & (kBN - 1), h = u >> 7;
         const unsigned full = 0xffffffffu;
         bool ok = true;
         for (int r = 0; r < nr && ok; ++r) {
@@ -253,12 +271,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint8_t* rbase = r_ring + rs * RT::bytes + t * 128;
             const uint4 sv = lds128(s_ring + rs * kScaleTile + t * 16);
             const uint32_t sw[4] = {sv.x, sv.y, sv.z, sv.w};
-            float d[8], nbd[8];
+            float d[4], nbd[4];  // scale of block 2j + h (word j, half h), j = 0..3
 #pragma unroll
-            for (int b = 0; b < 8; ++b) {
-                const uint16_t hb = uint16_t((sw[b >> 1] >> (16 * (b & 1))) & 0xFFFFu);
-                d[b] = __half2float(__ushort_as_half(hb));
-                nbd[b] = -RT::bias * d[b];  // exact (see bytes_to_w)
+            for (int j = 0; j < 4; ++j) {
+                const uint16_t hb = uint16_t((sw[j] >> (16 * h)) & 0xFFFFu);
+                d[j] = __half2float(__ushort_as_half(hb));
+                nbd[j] = -RT::bias * d[j];  // exact (see bytes_to_w)
             }
 #pragma unroll
             for (int j = 0; j < kStepsPerRaw; ++j) {
@@ -273,15 +291,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 uint8_t* arow = a_ring + s * kAT * kATile + t * 128;
                 const int sx = t & 7;  // 128B swizzle: 16-byte chunk c of row t lives at c ^ (t & 7)
                 if constexpr (FMT == EMB_Q8_0) {
-                    // atom j: codes 64j..64j+63 of the raw stage = plane j/2, chunks 4(j%2)..+3
+                    // atom j: codes 64j..64j+63 of the raw stage = plane j/2, chunks 4(j%2)..+3;
+                    // this half: chunks 4(j%2)+2h, +1 (block 2j+h) -> output chunks 4h..4h+3
 #pragma unroll
-                    for (int cc = 0; cc < 4; ++cc) {
+                    for (int cc = 2 * h; cc < 2 * h + 2; ++cc) {
                         const int c = (j & 1) * 4 + cc;
                         const uint4 v = lds128(rbase + (j >> 1) * kPlane + ((c ^ sx) << 4));
-                        const int b = 2 * j + (cc >> 1);  // 32-block within the raw stage
                         uint4 h0, l0, h1, l1;
-                        make_chunk<SPLIT>(v.x ^ 0x80808080u, v.y ^ 0x80808080u, d[b], nbd[b], h0, l0);
-                        make_chunk<SPLIT>(v.z ^ 0x80808080u, v.w ^ 0x80808080u, d[b], nbd[b], h1, l1);
+                        make_chunk<SPLIT>(v.x ^ 0x80808080u, v.y ^ 0x80808080u, d[j], nbd[j], h0, l0);
+                        make_chunk<SPLIT>(v.z ^ 0x80808080u, v.w ^ 0x80808080u, d[j], nbd[j], h1, l1);
                         const int o0 = 2 * cc, o1 = 2 * cc + 1;
                         sts128(arow + ((o0 ^ sx) << 4), h0);
                         sts128(arow + ((o1 ^ sx) << 4), h1);
@@ -291,24 +309,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         }
                     }
                 } else {
-                    // atom j: blocks 2j, 2j+1 = 16-byte chunks 2j, 2j+1 of the single plane;
-                    // a block's byte i holds code i (low nibble) and code i+16 (high nibble)
+                    // atom j: blocks 2j, 2j+1; this half: block 2j+h -> output chunks 4h..4h+3.
+                    // A block's byte i holds code i (low nibble) and code i+16 (high nibble).
+                    const int b = 2 * j + h;
+                    const uint4 v = lds128(rbase + ((b ^ sx) << 4));
+                    const uint32_t m = 0x0F0F0F0Fu;
+                    uint4 hh[4], ll[4];
+                    make_chunk<SPLIT>(v.x & m, v.y & m, d[j], nbd[j], hh[0], ll[0]);               // codes 0..7
+                    make_chunk<SPLIT>(v.z & m, v.w & m, d[j], nbd[j], hh[1], ll[1]);               // 8..15
+                    make_chunk<SPLIT>((v.x >> 4) & m, (v.y >> 4) & m, d[j], nbd[j], hh[2], ll[2]); // 16..23
+                    make_chunk<SPLIT>((v.z >> 4) & m, (v.w >> 4) & m, d[j], nbd[j], hh[3], ll[3]); // 24..31
 #pragma unroll
-                    for (int bb = 0; bb < 2; ++bb) {
-                        const int b = 2 * j + bb;
-                        const uint4 v = lds128(rbase + ((b ^ sx) << 4));
-                        const uint32_t m = 0x0F0F0F0Fu;
-                        uint4 h[4], l[4];
-                        make_chunk<SPLIT>(v.x & m, v.y & m, d[b], nbd[b], h[0], l[0]);               // codes 0..7
-                        make_chunk<SPLIT>(v.z & m, v.w & m, d[b], nbd[b], h[1], l[1]);               // 8..15
-                        make_chunk<SPLIT>((v.x >> 4) & m, (v.y >> 4) & m, d[b], nbd[b], h[2], l[2]); // 16..23
-                        make_chunk<SPLIT>((v.z >> 4) & m, (v.w >> 4) & m, d[b], nbd[b], h[3], l[3]); // 24..31
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const int o = 4 * bb + q;
-                            sts128(arow + ((o ^ sx) << 4), h[q]);
-                            if constexpr (SPLIT) sts128(arow + kATile + ((o ^ sx) << 4), l[q]);
-                        }
+                    for (int q = 0; q < 4; ++q) {
+                        const int o = 4 * h + q;
+                        sts128(arow + ((o ^ sx) << 4), hh[q]);
+                        if constexpr (SPLIT) sts128(arow + kATile + ((o ^ sx) << 4), ll[q]);
                     }
                 }
                 ptx::fence_proxy_async_smem();
@@ -325,27 +340,75 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         ok = __all_sync(full, ok && ptx::mbar_wait(acc_full, 0, abort_flag, p.status, kWaitLimitNs));
         if (ok) {
             ptx::tc_fence_after();
-            const int quarter = warp & 3;  // TMEM lanes this warp may access
-            const int n = n0 + quarter * 32 + lane;
+            // warps 2..9: TMEM lane quarter = warp % 4; two warps per quarter split the columns
+            const int quarter = warp & 3, half = (warp - 2) >> 2;
+            const int csplit = ((T >> 1) + 15) & ~15;
+            const int cbeg = half ? csplit : 0, cend = half ? T : min(csplit, T);
+            const int row = quarter * 32 + lane;
             const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16);
+            const int n = n0 + row;
             float* Y = p.Y[g];
-            for (int c0 = 0; c0 < T; c0 += 16) {
+            for (int c0 = cbeg; c0 < cend; c0 += 16) {
                 uint32_t v[16];
                 ptx::tmem_ld_16(taddr + uint32_t(c0), v);
                 ptx::tmem_ld_wait();
-                if (n < N) {
+                if (splits == 1) {
+                    if (n < N) {
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const int m = m0 + c0 + e;
-                        if (m < M) Y[int64_t(m) * N + n] = __uint_as_float(v[e]);
+                        for (int e = 0; e < 16; ++e) {
+                            const int m = m0 + c0 + e;
+                            if (m < M) Y[int64_t(m) * N + n] = __uint_as_float(v[e]);
+                        }
                     }
+                } else {
+                    // token-major partial tile part[m][row] (a warp writes 32 consecutive rows)
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) part[(c0 + e) * kBN + row] = __uint_as_float(v[e]);
                 }
             }
         }
     }
 
+    __syncwarp();  // the producer / MMA warps reconverge before the block-wide barriers
     ptx::tc_fence_before();
-    __syncthreads();
+    if (splits > 1) {
+        // split-K: every CTA of the cluster holds its partial tile; CTA s sums rows
+        // [s*128/splits, (s+1)*128/splits) over the cluster in a fixed order through
+        // distributed shared memory and stores them (deterministic, no global scratch)
+        ptx::cluster_sync();
+        if (threadIdx.x >= 64 && !*abort_flag) {
+            // one thread = 4 consecutive rows of one token: 16-byte remote loads and
+            // 16-byte coalesced stores to Y[m][n..n+3]
+            const int rows = kBN / splits, r0 = split * rows, q4 = rows / 4;
+            const uint32_t pbase = ptx::smem_u32(part);
+            float* Y = p.Y[g];
+            const bool vec = (N % 4) == 0;
+            for (int w = threadIdx.x - 64; w < q4 * T; w += kThreads - 64) {
+                const int c = w / q4, row = r0 + 4 * (w - c * q4);
+                const int m = m0 + c, n = n0 + row;
+                const uint32_t off = pbase + uint32_t(c * kBN + row) * 4u;
+                float4 acc = ptx::ld_dsmem_f32x4(ptx::map_dsmem(off, 0));
+                for (int q = 1; q < splits; ++q) {
+                    const float4 v = ptx::ld_dsmem_f32x4(ptx::map_dsmem(off, q));
+                    acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+                }
+                if (m < M) {
+                    float* dst = Y + int64_t(m) * N + n;
+                    if (vec && n + 3 < N) {
+                        *reinterpret_cast<float4*>(dst) = acc;
+                    } else {
+                        if (n < N) dst[0] = acc.x;
+                        if (n + 1 < N) dst[1] = acc.y;
+                        if (n + 2 < N) dst[2] = acc.z;
+                        if (n + 3 < N) dst[3] = acc.w;
+                    }
+                }
+            }
+        }
+        ptx::cluster_sync();  // remote shared memory must outlive its readers
+    } else {
+        __syncthreads();
+    }
     if (warp == 1) {
         __syncwarp();
         ptx::tc_fence_after();
@@ -405,6 +468,8 @@ int pick_stages(int T) {
 
 template <int FMT, bool SPLIT>
 cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl, cudaStream_t s) {
+    // grid: x = token tile (fastest, so the CTAs sharing a weight tile run together and
+    // read it from L2 after the first), y = weight-row tile, z = K split (one cluster)
     const int bytes = smem_bytes<FMT, SPLIT>(p.T, p.stages);
     // the opt-in shared-memory size is a per-device function attribute
     static std::mutex mu;
@@ -422,16 +487,47 @@ cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl,
         }
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(grid_x, grid_y, 1);
+    cfg.gridDim = dim3(grid_x, grid_y, p.splits);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = size_t(bytes);
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    if (pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
+    if (p.splits > 1) {
+        attr[na].id = cudaLaunchAttributeClusterDimension;
+        attr[na].val.clusterDim.x = 1;
+        attr[na].val.clusterDim.y = 1;
+        attr[na].val.clusterDim.z = unsigned(p.splits);
+        ++na;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
+    cfg.numAttrs = na;
     return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<FMT, SPLIT>, p);
+}
+
+// K splits (1, 2 or 4; one cluster of CTAs per output tile): the count minimising a
+// simple time model -- waves of 148 CTAs, each costing a fixed ~3 us plus its share of the
+// tile's MMA work at ~11.6 TFLOP/s per SM -- subject to every split owning at least one
+// 256-k raw stage and the partial tile fitting in the CTA's A/X rings.
+int pick_splits(int64_t tiles, int T, int64_t K, int stages, bool split_operand) {
+    const int64_t nr = (K + kKR - 1) / kKR;
+    const double work_us = 2.0 * kBN * T * double(K) / 11.6e12 * 1e6 * (split_operand ? 2 : 1);
+    const int64_t ring = int64_t(stages) * ((split_operand ? 2 : 1) * kATile + int64_t(T) * 128);
+    const int64_t part = int64_t(kBN) * T * 4;
+    int best = 1;
+    double best_t = 1e30;
+    for (int sp = 1; sp <= 4; sp *= 2) {
+        if (sp > nr || (sp > 1 && part > ring)) break;
+        const int64_t ctas = tiles * sp;
+        const double t = double((ctas + 147) / 148) * (3.0 + work_us / sp);
+        if (t < best_t * 0.97) { best_t = t; best = sp; }
+    }
+    return best;
 }
 
 }  // namespace
@@ -477,16 +573,17 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.K = int32_t(g.K);
     p.T = T;
     p.stages = S;
+    p.splits = pick_splits(int64_t(t_tiles) * tiles, T, g.K, S, split);
     uint32_t cols = 32;
     while (cols < uint32_t(T)) cols <<= 1;
     p.tmem_cols = cols;
     p.status = status;
-    const int grid_y = int(t_tiles);
+    const int grid_x = int(t_tiles);
     if (g.fmt == EMB_Q8_0)
-        return split ? launch_kernel<EMB_Q8_0, true>(p, tiles, grid_y, pdl, s)
-                     : launch_kernel<EMB_Q8_0, false>(p, tiles, grid_y, pdl, s);
-    return split ? launch_kernel<EMB_Q4_0, true>(p, tiles, grid_y, pdl, s)
-                 : launch_kernel<EMB_Q4_0, false>(p, tiles, grid_y, pdl, s);
+        return split ? launch_kernel<EMB_Q8_0, true>(p, grid_x, tiles, pdl, s)
+                     : launch_kernel<EMB_Q8_0, false>(p, grid_x, tiles, pdl, s);
+    return split ? launch_kernel<EMB_Q4_0, true>(p, grid_x, tiles, pdl, s)
+                 : launch_kernel<EMB_Q4_0, false>(p, grid_x, tiles, pdl, s);
 }
 
 }  // namespace emb
