@@ -454,12 +454,16 @@ def run_ours(args):
 def kernel_traffic(workload, w):
     """DRAM bytes per launch of the dominant kernel from the committed ncu summary, if
     one exists for this workload and matches the current kernel build."""
+    import hashlib
     path = os.path.join(ROOT, "profiles", f"traffic_{workload}.json")
     try:
         with open(path) as fh:
             d = json.load(fh)
+        with open(os.path.join(ROOT, d["source"]), "rb") as fh:
+            if hashlib.sha256(fh.read()).hexdigest() != d["source_sha256"]:
+                return None   # the kernel changed since the counters were taken
         return d.get(wl.FMT_NAMES[w.fmt])
-    except (OSError, ValueError):
+    except (OSError, ValueError, KeyError):
         return None
 
 
