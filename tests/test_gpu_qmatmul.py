@@ -95,3 +95,37 @@ def test_y_fully_overwritten(cuda_device):
             emb.qmatmul(fmt, img, X, N, out=Y1)
             torch.cuda.synchronize()
             assert torch.equal(Y0, Y1)
+
+
+# Layers of at least 12 MB of packed weights take the staged (bulk-copy ring) GEMV: ragged
+# row counts (partial last tile and partial last run of tiles per CTA), K not a multiple of
+# the warps' K slices, M = 1..4 and the largest staged activation row (K = 16384 at M = 1).
+STAGED_SHAPES = [(1, 24593, 1056), (2, 6151, 4128), (3, 6151, 4096), (4, 12301, 2048),
+                 (1, 1543, 16384), (1, 12289, 2048)]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("M,N,K", STAGED_SHAPES)
+def test_staged_gemv_parity(cuda_device, fmt, M, N, K):
+    Y, Yref, B, _, _ = run_case(fmt, M, N, K, seed=M * 5 + N + K)
+    check_close(Y, Yref, B, f"staged gemv fmt={fmt} M={M} N={N} K={K}")
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_staged_gemv_fused_group(cuda_device, fmt):
+    """Two matrices sharing X in one launch (gate/up): tiles of both in one CTA's run."""
+    M, K, Ns = 1, 2048, (12289, 12291)
+    Xb = activation_bits_np(M, K, 31)
+    X = to_dev_bf16(Xb)
+    specs, host = [], []
+    for i, N in enumerate(Ns):
+        W = weight_np(N, K, 40 + i)
+        img = emb.quantize(fmt, torch.from_numpy(W).cuda())
+        Y = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+        specs.append((fmt, img, N, K, X, Y))
+        host.append(W)
+    emb.emb_qlayer_seq(specs, M)
+    torch.cuda.synchronize()
+    for (f, img, N, _, _, Y), W in zip(specs, host):
+        Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
+        check_close(Y.cpu().numpy(), Yref, B, f"fused staged N={N}")
