@@ -2,7 +2,7 @@
 //
 // The paper's batch-1 setting (Section 3.1, challenge 2) makes every linear layer a
 // matrix-vector product whose cost is reading the packed weights once from HBM.
-// Two kernels share the dequantise-and-dot arithmetic below:
+// Three kernels:
 //   * the staged kernel (large layers with short rows, and M > 1): each CTA pulls one
 //     tile of rows plus its activations into shared memory with cp.async.bulk, so many
 //     bytes are in flight per SM and the next layer's tiles load during this layer's
@@ -12,10 +12,12 @@
 //     16 codes, half a block; a Q4_0 unit is one whole 32-code block; a warp reads 512
 //     contiguous bytes), load codes with 128-bit non-allocating loads one unit ahead
 //     (register double buffering) and reduce with warp shuffles, then across warps in
-//     shared memory.
-// Both dequantise in registers with exact integer->float "magic number" conversions
-// followed by packed fp32x2 FMAs (FFMA2); reductions run in a fixed order, so results
-// are deterministic. Weights are fetched before griddepcontrol.wait (they never depend
+//     shared memory;
+//   * the Q4_0 tensor-core kernel (large Q4_0 layers at M = 2..8): staged like the
+//     first, with the dot products on mma.sync (described at its definition).
+// The first two dequantise in registers with exact integer->float "magic number"
+// conversions followed by packed fp32x2 FMAs (FFMA2). Every reduction runs in a fixed
+// order, so results are deterministic. Weights are fetched before griddepcontrol.wait (they never depend
 // on an earlier launch); X is read and Y written only after it.
 // Up to kMaxGroup matrices that read the same X (q/k/v or gate/up) share one launch.
 #include <mutex>
@@ -53,7 +55,15 @@ __device__ __forceinline__ void griddep_launch_dependents() {
 
 __device__ __forceinline__ float lo_bf16(uint32_t h) { return __uint_as_float(h << 16); }
 __device__ __forceinline__ float hi_bf16(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
-__device__ __forceinline__ float magic(uint32_t bits) { return __uint_as_float(bits | 0x4B000000u); }
+// (a & mask) | bits in one LOP3 (written out: the compiler otherwise emits an AND and
+// an OR when both constants are immediates).
+__device__ __forceinline__ uint32_t and_or(uint32_t a, uint32_t mask, uint32_t bits) {
+    uint32_t d;
+    asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(d) : "r"(a), "r"(mask), "r"(bits));
+    return d;
+}
+// Nibble field of v selected by mask, as the binary32 2^23 + field (exact).
+__device__ __forceinline__ float magic(uint32_t v, uint32_t mask) { return __uint_as_float(and_or(v, mask, 0x4B000000u)); }
 
 // 16 Q8_0 codes (one unit) times 16 fp32 activations -> fp32 partial sum.
 // __byte_perm(v ^ 0x80808080, 0x4B000000, 0x7540 + i) is the binary32 2^23 + (q_i + 128)
@@ -93,13 +103,13 @@ __device__ __forceinline__ float dot_q4_unit(const uint4 c, const float* x) {
     for (int j = 0; j < 4; ++j) {
         const uint32_t v = w[j], v2 = w[j] >> 12;
         // codes 4j, 4j+1 (bits 0..3, 8..11)
-        const float2 a = __ffma2_rn(make_float2(magic(v & 0xFu), magic(v & 0xF00u)), s_a, o_a);
+        const float2 a = __ffma2_rn(make_float2(magic(v, 0xFu), magic(v, 0xF00u)), s_a, o_a);
         // codes 16+4j, 16+4j+1 (bits 4..7, 12..15)
-        const float2 b = __ffma2_rn(make_float2(magic(v & 0xF0u), magic(v & 0xF000u)), s_b, o_b);
+        const float2 b = __ffma2_rn(make_float2(magic(v, 0xF0u), magic(v, 0xF000u)), s_b, o_b);
         // codes 4j+2, 4j+3 (bits 16..19, 24..27 -> 12..15 after the shift)
-        const float2 cc = __ffma2_rn(make_float2(magic(v & 0xF0000u), magic(v2 & 0xF000u)), s_c, o_c);
+        const float2 cc = __ffma2_rn(make_float2(magic(v, 0xF0000u), magic(v2, 0xF000u)), s_c, o_c);
         // codes 16+4j+2, 16+4j+3 (bits 20..23 -> 8..11, 28..31 -> 16..19)
-        const float2 d = __ffma2_rn(make_float2(magic(v2 & 0xF00u), magic(v2 & 0xF0000u)), s_d, o_d);
+        const float2 d = __ffma2_rn(make_float2(magic(v2, 0xF00u), magic(v2, 0xF0000u)), s_d, o_d);
         acc = __ffma2_rn(a, make_float2(x[4 * j + 0], x[4 * j + 1]), acc);
         acc = __ffma2_rn(cc, make_float2(x[4 * j + 2], x[4 * j + 3]), acc);
         acc = __ffma2_rn(b, make_float2(x[16 + 4 * j + 0], x[16 + 4 * j + 1]), acc);
@@ -511,12 +521,250 @@ bool launch_staged(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     return true;
 }
 
+
+// ------------------------------------------------------------ Q4_0 tensor-core GEMV
+// For Q4_0 the dequantise-and-dot arithmetic, not HBM, bounds the kernels above. Here
+// the dot products run on the tensor cores (mma.sync m16n8k16, bf16 x bf16 -> fp32) and
+// the CUDA cores only unpack nibbles: a nibble OR-ed into the bf16 pattern 0x4300 is
+// 128 + q exactly, and one packed bf16 subtraction of 136 leaves q - 8 exactly, so each
+// pair of weights costs one LOP3 and one HSUB2. One MMA covers 16 rows x 16 consecutive
+// K of one block (the tokens, M <= 8, are the MMA's 8 columns); a block's two MMAs
+// accumulate into a fresh fragment that is then scaled by the block's fp32 scale, as in
+// the plain definition. The MMA sums its 16 products in its own fixed order, so results
+// are deterministic.
+//
+// Fragment mapping (any permutation of K inside a block is valid as long as A and B use
+// the same one): lane (g, t) = (lane / 4, lane % 4) loads 32-bit word t of the block in
+// rows g and g + 8. Word t holds q[4t + i] in the low nibble and q[16 + 4t + i] in the
+// high nibble of its byte i. MMA 0 takes the low nibbles: (bytes 0, 2) -> k slots
+// (2t, 2t + 1), (bytes 1, 3) -> (2t + 8, 2t + 9); MMA 1 the high nibbles likewise. The
+// activation fragment of lane (g, t) is token g's x at the same four positions.
+//
+// The CTA's tile (TR rows, TR a multiple of 16) and its activations are staged in shared
+// memory as in the staged kernel, but row by row into a padded layout (pitch = row
+// bytes + 16) so that the eight rows a fragment load touches fall into distinct banks.
+constexpr int kMmaWarps = 4;
+constexpr int kMmaThreads = 32 * kMmaWarps;
+constexpr int kMmaTileBytes = 32 * 1024;  // codes of one tile, at most
+constexpr int kMmaMaxM = 8;
+constexpr int kMmaHeader = 128 + 512 * 4;  // barriers, then cross-warp sums [WK][TR][8] (WK * TR <= 64)
+
+struct MmaParams {
+    const uint8_t* codes[kMaxGroup];
+    const __half* scales[kMaxGroup];
+    float* Y[kMaxGroup];
+    int32_t N[kMaxGroup];
+    int32_t tile0[kMaxGroup + 1];
+    int32_t n_mats;
+    int32_t M, K, ldS;
+    int32_t TR, WK;                // rows per tile (multiple of 16), warps along K
+    int32_t pitch, spitch;         // padded shared-memory row pitch of codes / scales, bytes
+    const __nv_bfloat16* X;
+    int* status;
+};
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%10, %11, %12, %13};"
+        : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.0f), "f"(0.0f), "f"(0.0f),
+          "f"(0.0f));
+}
+
+// (128 + q) pairs from the nibbles at bits 0..3 and 16..19, then q - 8 (exact in bf16).
+__device__ __forceinline__ uint32_t q4_pair(uint32_t v) {
+    const uint32_t b = and_or(v, 0x000F000Fu, 0x43004300u);
+    const __nv_bfloat162 r = __hsub2(*reinterpret_cast<const __nv_bfloat162*>(&b),
+                                     __floats2bfloat162_rn(136.0f, 136.0f));
+    return *reinterpret_cast<const uint32_t*>(&r);
+}
+
+__global__ void __launch_bounds__(kMmaThreads) gemv_q4_mma_kernel(const __grid_constant__ MmaParams p) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    uint64_t* bar_w = reinterpret_cast<uint64_t*>(smem);
+    uint64_t* bar_x = reinterpret_cast<uint64_t*>(smem + 8);
+    float* red = reinterpret_cast<float*>(smem + 128);  // [WK][TR][8]
+    const int row_bytes = p.K / 2;
+    const int nb = p.K / kQBlock;
+    uint8_t* x_s = smem + kMmaHeader;                  // [M][K] bf16
+    uint8_t* codes_s = x_s + p.M * p.K * 2;            // [TR][pitch]
+    uint8_t* scales_s = codes_s + p.TR * p.pitch;
+
+    const int tile = blockIdx.x;
+    int g_mat = 0;
+#pragma unroll
+    for (int i = 1; i < kMaxGroup; ++i)
+        if (i < p.n_mats && tile >= p.tile0[i]) g_mat = i;
+    const int N = p.N[g_mat];
+    const int row0 = (tile - p.tile0[g_mat]) * p.TR;
+    const int rows = min(p.TR, N - row0);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            ptx::mbar_init(bar_w, 1);
+            ptx::mbar_init(bar_x, 1);
+            ptx::fence_mbar_init();
+            ptx::mbar_arrive_expect_tx(bar_w, uint32_t(rows) * uint32_t(row_bytes + p.ldS * 2));
+        }
+        __syncwarp();
+        const uint8_t* src_c = p.codes[g_mat] + int64_t(row0) * row_bytes;
+        const __half* src_s = p.scales[g_mat] + int64_t(row0) * p.ldS;
+        for (int r = lane; r < rows; r += 32) {
+            ptx::bulk_load(codes_s + r * p.pitch, src_c + int64_t(r) * row_bytes, uint32_t(row_bytes), bar_w);
+            ptx::bulk_load(scales_s + r * p.spitch, src_s + int64_t(r) * p.ldS, uint32_t(p.ldS * 2), bar_w);
+        }
+    }
+    ptx::griddep_launch_dependents();
+    // weights do not depend on earlier launches; X and Y may
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) {
+        const uint32_t x_bytes = uint32_t(p.M) * uint32_t(p.K) * 2u;
+        ptx::mbar_arrive_expect_tx(bar_x, x_bytes);
+        ptx::bulk_load(x_s, p.X, x_bytes, bar_x);
+    }
+    __syncthreads();  // the barriers' initialisation is visible to every waiting thread
+    // both waits are bounded; the CTA leaves together if any of its threads gave up
+    bool ok = ptx::mbar_wait(bar_w, 0, nullptr, p.status, kWaitLimitNs);
+    ok = ok && ptx::mbar_wait(bar_x, 0, nullptr, p.status, kWaitLimitNs);
+    if (__syncthreads_or(!ok)) return;
+
+    const int WK = p.WK;
+    const int wk = warp % WK, rg = warp / WK;  // K slice, 16-row group
+    const int gq = lane >> 2, t = lane & 3;
+    const int bw = (nb + WK - 1) / WK;
+    const int kb_lo = wk * bw, kb_hi = min(nb, kb_lo + bw);
+    const uint8_t* c0 = codes_s + (rg * 16 + gq) * p.pitch + 4 * t;
+    const uint8_t* c1 = c0 + 8 * p.pitch;
+    const __half* s0 = reinterpret_cast<const __half*>(scales_s + (rg * 16 + gq) * p.spitch);
+    const __half* s1 = reinterpret_cast<const __half*>(reinterpret_cast<const uint8_t*>(s0) + 8 * p.spitch);
+    const bool has_x = gq < p.M;
+    const uint8_t* xr = x_s + (gq * p.K + 4 * t) * 2;
+
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (rg * 16 < rows) {
+#pragma unroll 4
+        for (int kb = kb_lo; kb < kb_hi; ++kb) {
+            uint32_t b[4] = {0u, 0u, 0u, 0u};
+            if (has_x) {
+                const uint2 lo = *reinterpret_cast<const uint2*>(xr + kb * 64);       // x[4t .. 4t+3]
+                const uint2 hi = *reinterpret_cast<const uint2*>(xr + kb * 64 + 32);  // x[16+4t ..]
+                b[0] = __byte_perm(lo.x, lo.y, 0x5410);
+                b[1] = __byte_perm(lo.x, lo.y, 0x7632);
+                b[2] = __byte_perm(hi.x, hi.y, 0x5410);
+                b[3] = __byte_perm(hi.x, hi.y, 0x7632);
+            }
+            const uint32_t w0 = *reinterpret_cast<const uint32_t*>(c0 + kb * 16);
+            const uint32_t w1 = *reinterpret_cast<const uint32_t*>(c1 + kb * 16);
+            const uint32_t alo[4] = {q4_pair(w0), q4_pair(w1), q4_pair(w0 >> 8), q4_pair(w1 >> 8)};
+            const uint32_t ahi[4] = {q4_pair(w0 >> 4), q4_pair(w1 >> 4), q4_pair(w0 >> 12), q4_pair(w1 >> 12)};
+            float dlo[4], dhi[4];
+            mma_bf16_16816(dlo, alo, b[0], b[1]);
+            mma_bf16_16816(dhi, ahi, b[2], b[3]);
+            const float sc0 = __half2float(s0[kb]), sc1 = __half2float(s1[kb]);
+            acc[0] = fmaf(sc0, dlo[0] + dhi[0], acc[0]);
+            acc[1] = fmaf(sc0, dlo[1] + dhi[1], acc[1]);
+            acc[2] = fmaf(sc1, dlo[2] + dhi[2], acc[2]);
+            acc[3] = fmaf(sc1, dlo[3] + dhi[3], acc[3]);
+        }
+    }
+    // acc[0], acc[1]: row gq, tokens 2t, 2t+1; acc[2], acc[3]: row gq + 8, same tokens
+    const int ra = rg * 16 + gq, rb = ra + 8, m0 = 2 * t;
+    float* Yg = p.Y[g_mat];
+    if (WK == 1) {
+        if (m0 < p.M) {
+            if (ra < rows) Yg[int64_t(m0) * N + row0 + ra] = acc[0];
+            if (rb < rows) Yg[int64_t(m0) * N + row0 + rb] = acc[2];
+        }
+        if (m0 + 1 < p.M) {
+            if (ra < rows) Yg[int64_t(m0 + 1) * N + row0 + ra] = acc[1];
+            if (rb < rows) Yg[int64_t(m0 + 1) * N + row0 + rb] = acc[3];
+        }
+        return;
+    }
+    float* rw = red + wk * p.TR * 8;
+    rw[ra * 8 + m0] = acc[0];
+    rw[ra * 8 + m0 + 1] = acc[1];
+    rw[rb * 8 + m0] = acc[2];
+    rw[rb * 8 + m0 + 1] = acc[3];
+    __syncthreads();
+    // add the K slices in slice order
+    for (int e = threadIdx.x; e < rows * p.M; e += kMmaThreads) {
+        const int r = e / p.M, m = e % p.M;
+        float v = 0.0f;
+        for (int k = 0; k < WK; ++k) v += red[(k * p.TR + r) * 8 + m];
+        Yg[int64_t(m) * N + row0 + r] = v;
+    }
+}
+
+// Q4_0 layers with 2..8 tokens, large enough for the staged path and with rows of at
+// most 2 KB (K <= 4096). At M = 1 the FFMA2 staged kernel is faster (measured on GB300,
+// Q4_0 32768 x 2048: 13.0 us FFMA2, 16.4 us MMA); from M = 2 the MMA's cost does not grow
+// with the token count while FFMA2's does (M = 4: 17.0 us MMA, 29.5 us FFMA2).
+// TR = 32 rows (2 row groups x 2 K slices) when that still gives 4 tiles per SM, else
+// 16 rows (4 K slices).
+bool launch_q4_mma(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
+    if (g.fmt != EMB_Q4_0 || g.M < 2 || g.M > kMmaMaxM) return false;
+    const int64_t row_bytes = g.K / 2;
+    if (row_bytes * 16 > kMmaTileBytes) return false;
+    if (g.M * g.K * 2 > kStageXBytes) return false;
+    int64_t rows = 0;
+    for (int i = 0; i < g.n_mats; ++i) rows += g.mats[i].N;
+    if (rows * row_bytes < kStageMinBytes) return false;
+    const int nb = int(g.K / kQBlock);
+    int TR = 16, WK = 4;
+    if (row_bytes * 32 <= kMmaTileBytes && rows / 32 >= 4 * 152) { TR = 32; WK = 2; }
+    if (nb < WK) WK = 1, TR = 16 * kMmaWarps;  // too few blocks to split K: 4 row groups
+    if (TR * row_bytes > kMmaTileBytes) return false;
+    MmaParams p = {};
+    int tiles = 0;
+    for (int i = 0; i < g.n_mats; ++i) {
+        p.codes[i] = g.mats[i].codes;
+        p.scales[i] = g.mats[i].scales;
+        p.Y[i] = g.mats[i].Y;
+        p.N[i] = int32_t(g.mats[i].N);
+        p.tile0[i] = tiles;
+        tiles += int((g.mats[i].N + TR - 1) / TR);
+    }
+    p.tile0[g.n_mats] = tiles;
+    p.n_mats = g.n_mats;
+    p.M = int32_t(g.M);
+    p.K = int32_t(g.K);
+    p.ldS = int32_t(g.ldS);
+    p.TR = TR;
+    p.WK = WK;
+    p.pitch = int32_t(row_bytes + 16);
+    p.spitch = int32_t(g.ldS * 2 + 16);
+    p.X = g.X;
+    p.status = status;
+    const size_t smem = size_t(kMmaHeader) + size_t(g.M) * g.K * 2 + size_t(TR) * (p.pitch + p.spitch);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(tiles, 1, 1);
+    cfg.blockDim = dim3(kMmaThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    if (smem > 48 * 1024) {
+        err = cudaFuncSetAttribute(gemv_q4_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        if (err != cudaSuccess) return true;
+    }
+    err = cudaLaunchKernelEx(&cfg, gemv_q4_mma_kernel, p);
+    return true;
+}
+
 }  // namespace
 
 cudaError_t launch_gemv_regs(const GroupRef& g, bool pdl, cudaStream_t s);
 
 cudaError_t launch_gemv(const GroupRef& g, bool pdl, int* status, cudaStream_t s) {
     cudaError_t err = cudaSuccess;
+    if (launch_q4_mma(g, pdl, status, s, err)) return err;
     if (launch_staged(g, pdl, status, s, err)) return err;
     return launch_gemv_regs(g, pdl, s);
 }

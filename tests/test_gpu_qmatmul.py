@@ -101,7 +101,7 @@ def test_y_fully_overwritten(cuda_device):
 # row counts (partial last tile and partial last run of tiles per CTA), K not a multiple of
 # the warps' K slices, M = 1..4 and the largest staged activation row (K = 16384 at M = 1).
 STAGED_SHAPES = [(1, 24593, 1056), (2, 6151, 4128), (3, 6151, 4096), (4, 12301, 2048),
-                 (1, 1543, 16384), (1, 12289, 2048)]
+                 (1, 1543, 16384), (1, 12289, 2048), (2, 12289, 2048), (1, 6151, 4096)]
 
 
 @pytest.mark.parametrize("fmt", FMTS)
@@ -126,6 +126,11 @@ def test_staged_gemv_fused_group(cuda_device, fmt):
         host.append(W)
     emb.emb_qlayer_seq(specs, M)
     torch.cuda.synchronize()
+    first = [sp[5].clone() for sp in specs]
+    emb.emb_qlayer_seq(specs, M)
+    torch.cuda.synchronize()
+    for a, sp in zip(first, specs):
+        assert torch.equal(a.view(torch.int32), sp[5].view(torch.int32))   # deterministic
     for (f, img, N, _, _, Y), W in zip(specs, host):
         Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
         check_close(Y.cpu().numpy(), Yref, B, f"fused staged N={N}")
