@@ -421,8 +421,8 @@ def run_ours(args):
                 "peak_source": f"{peaks['source']} HBM copy bandwidth"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["traffic"] = kernel_traffic(args.workload, c["w"])
-    roof["kernel"] = ("gemv_kernel" if c["w"].M <= 4 else "gemm_tc_kernel") + \
-        f"<{wl.FMT_NAMES[c['w'].fmt]}>"
+    roof["kernel"] = ("GEMV (gemv_staged_kernel + gemv_kernel + gemv_q4_mma_kernel)" if c["w"].M <= 4
+                      else "gemm_tc_kernel") + f" <{wl.FMT_NAMES[c['w'].fmt]}>"
     roof["launches_per_step"] = c["launches"] * c["w"].repeats
     roof["per_launch_us"] = per_launch_ms * 1e3
 

@@ -445,17 +445,24 @@ cudaError_t launch_staged_rw(const StagedParams& p, int RW, int tiles, size_t sm
 }
 
 // Tile shape: rows per warp RW and warps along K WK (TR = RW * 4 / WK rows per tile),
-// in order of preference (more rows per warp = more activation reuse). Take the first
-// whose tile fits kStageBytes and that makes at least 4 tiles per SM; for matrices too
-// small for that, the fitting shape with the most tiles. A warp's K slice keeps at least
-// 32 units (one per lane). Returns false when no tile fits (rows above kStageBytes).
-bool pick_stage_shape(int64_t rows_total, int64_t row_bytes, int U, int& RW, int& WK) {
-    static const int kShapes[5][2] = {{4, 1}, {4, 2}, {4, 4}, {2, 4}, {1, 4}};
+// in order of preference: Q8_0 favours activation reuse (4 rows per warp), Q4_0 unsplit
+// K. Take the first whose tile fits `tile_bytes` and that makes at least 4 tiles per
+// SM; for matrices too small for that, the fitting shape with the most tiles. A warp's
+// K slice keeps at least 32 units (one per lane). Returns false when no tile fits.
+// Measured on GB300 at M = 1 (graph-replayed chains): 16 KB tiles beat 32 KB ones by
+// 3-6% (a shorter CTA lifetime shortens each launch's tail), e.g. Q8_0 32768 x 2048:
+// 14.9 us (8 rows) vs 15.8 us (16 rows); at M = 4, 32 KB tiles win (22.7 vs 27.0 us).
+bool pick_stage_shape(int fmt, int64_t rows_total, int64_t row_bytes, int U, int64_t tile_bytes,
+                      int& RW, int& WK) {
+    static const int kQ8[5][2] = {{4, 1}, {4, 2}, {4, 4}, {2, 4}, {1, 4}};
+    static const int kQ4[7][2] = {{4, 1}, {2, 1}, {1, 1}, {4, 2}, {4, 4}, {2, 4}, {1, 4}};
+    const int n = (fmt == EMB_Q8_0) ? 5 : 7;
     bool found = false;
-    for (const auto& sh : kShapes) {
-        const int rw = sh[0], wk = sh[1];
+    for (int i = 0; i < n; ++i) {
+        const int rw = (fmt == EMB_Q8_0) ? kQ8[i][0] : kQ4[i][0];
+        const int wk = (fmt == EMB_Q8_0) ? kQ8[i][1] : kQ4[i][1];
         const int64_t tr = int64_t(rw) * kStageWarps / wk;
-        if (tr * row_bytes > kStageBytes) continue;
+        if (tr * row_bytes > tile_bytes) continue;
         if (wk > 1 && U / wk < 32) continue;
         RW = rw;
         WK = wk;
@@ -486,7 +493,8 @@ bool launch_staged(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     if (rows * row_bytes < kStageMinBytes) return false;
     if (g.M == 1 && row_bytes > kStageMaxRowBytesM1) return false;
     int RW = 0, WK = 0;
-    if (!pick_stage_shape(rows, row_bytes, U, RW, WK)) return false;
+    const int64_t tile_bytes = (g.M == 1) ? kStageBytes / 2 : kStageBytes;
+    if (!pick_stage_shape(g.fmt, rows, row_bytes, U, tile_bytes, RW, WK)) return false;
     StagedParams p = {};
     const int TR = RW * kStageWarps / WK;
     int tiles = 0;
