@@ -1,19 +1,27 @@
 // Tensor-core GEMM for the larger token counts of one closed-loop step (M = 50 action
 // chunk, M = 280..816 prefix prefill): packed Q8_0/Q4_0 weights are staged in shared
-// memory by TMA, dequantised by four warps into 128B-swizzled bf16 tiles, and fed to
-// tcgen05 MMAs whose fp32 accumulators live in TMEM.
+// memory by TMA, dequantised by eight warps into bf16 tiles held in tensor memory, and
+// fed to tcgen05 MMAs (A operand from TMEM, B from shared memory) whose fp32
+// accumulators also live in TMEM.
 //
 // "Swap AB": the MMA's M side is 128 weight rows (output features n), its N side is the
 // CTA's T tokens, so one weight tile is dequantised once for up to 256 tokens and the
 // accumulator D[n][m] sits in TMEM lanes = n. The epilogue reads TMEM lane n (one
 // thread per output feature) and writes Y[m][n] with 128-byte coalesced stores.
 //
+// TMEM (512 columns, one CTA per SM): columns 0..255 the accumulator, 256..511 the ring
+// of bf16 A tiles (32 columns = 64 k per tile, two values per column, row n in lane n).
+// Keeping A out of shared memory leaves shared-memory bandwidth to the X tiles (written
+// by TMA, read by the MMA), which bound this kernel (measured on GB300: 100 -> 70 KB of
+// shared-memory traffic per 64-k step; M = 816 prefill 683 -> 736 TFLOP/s).
+//
 // Roles (320 threads):
 //   warp 0 lane 0 : TMA producer. Raw stages (256 codes of 128 rows + their 8 scales)
 //                   are fetched before griddepcontrol.wait (weights never depend on
 //                   the previous launch); X tiles (64 k x T tokens) after it.
 //   warp 1        : TMEM allocation; lane 0 issues the MMAs (4 x K=16 per 64-k stage).
-//   warps 2..9    : dequantisation (two threads per weight row), then the epilogue.
+//   warps 2..9    : dequantisation (two threads per weight row, tcgen05.st into the
+//                   warp's lane quarter), then the epilogue.
 // Grid: x = token tile (fastest: CTAs sharing a weight tile run together), y = weight-row
 // tile, z = K split. With z > 1 the splits of one output tile form a thread-block cluster
 // and are summed in a fixed order through distributed shared memory (deterministic).
@@ -41,7 +49,9 @@ constexpr int kStepsPerRaw = kKR / kKC;    // 4
 constexpr int kRawStages = 2;
 constexpr int kDeqWarps = 8;               // dequantisation (then epilogue) warps
 constexpr int kThreads = 64 + 32 * kDeqWarps;
-constexpr int kATile = kBN * kKC * 2;      // 16 KB bf16 tile
+constexpr int kAccCols = 256;              // TMEM columns [0, 256): the fp32 accumulator (T <= 256)
+constexpr int kACols = kKC / 2;            // TMEM columns of one bf16 A tile (two values per column)
+constexpr uint32_t kTmemCols = 512;        // accumulator + A stages
 constexpr int kPlane = kBN * 128;          // 16 KB: 128 rows x 128 bytes of codes
 constexpr int kScaleTile = kBN * 16;       // 2 KB: 128 rows x 8 fp16 scales
 
@@ -72,7 +82,6 @@ struct RawTraits {
 __device__ __forceinline__ uint4 lds128(const uint8_t* p) {
     return *reinterpret_cast<const uint4*>(p);
 }
-__device__ __forceinline__ void sts128(uint8_t* p, uint4 v) { *reinterpret_cast<uint4*>(p) = v; }
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -122,8 +131,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
                                                ~uintptr_t(1023));
     const int S = p.stages, T = p.T;
-    uint8_t* a_ring = base;                                     // S x kAT x 16 KB
-    uint8_t* x_ring = a_ring + S * kAT * kATile;                // S x T x 128 B
+    uint8_t* x_ring = base;                                     // S x T x 128 B
     uint8_t* r_ring = x_ring + S * T * 128;                     // 2 x RT::bytes
     uint8_t* s_ring = r_ring + kRawStages * RT::bytes;          // 2 x 2 KB
     uint64_t* bars = reinterpret_cast<uint64_t*>(s_ring + kRawStages * kScaleTile);
@@ -135,9 +143,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint64_t* acc_full = ax_empty + S;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-    // split-K partial tile [T][128] fp32 (token-major): reuses the A/X rings once every
-    // MMA has completed
-    float* part = reinterpret_cast<float*>(a_ring);
+    // split-K partial tile [T][128] fp32 (token-major): reuses the X ring once every MMA
+    // has completed
+    float* part = reinterpret_cast<float*>(x_ring);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tile = blockIdx.y;
@@ -233,22 +241,20 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         if (lane == 0) {
             // ------------------------------------------------------------ MMA issuer
             const uint32_t idesc = ptx::idesc_bf16_f32(kBN, T);
-            const uint32_t a0 = ptx::smem_u32(a_ring), x0 = ptx::smem_u32(x_ring);
+            const uint32_t x0 = ptx::smem_u32(x_ring);
             for (int i = 0; i < nk; ++i) {
                 const int s = i % S;
                 const uint32_t ph = (i / S) & 1;
                 if (!ptx::mbar_wait(&x_full[s], ph, abort_flag, p.status, kWaitLimitNs)) break;
                 if (!ptx::mbar_wait(&a_full[s], ph, abort_flag, p.status, kWaitLimitNs)) break;
                 ptx::tc_fence_after();
-                const uint32_t a_addr = a0 + s * kAT * kATile, x_addr = x0 + s * T * 128;
+                const uint32_t a_tm = tmem + uint32_t(kAccCols + s * kAT * kACols);
+                const uint32_t x_addr = x0 + s * T * 128;
 #pragma unroll
                 for (int k = 0; k < kKC / 16; ++k) {
                     const uint64_t bdesc = ptx::smem_desc_sw128(x_addr + 32 * k);
-                    ptx::mma_bf16(tmem, ptx::smem_desc_sw128(a_addr + 32 * k), bdesc, idesc,
-                                  (i | k) != 0);
-                    if constexpr (SPLIT)
-                        ptx::mma_bf16(tmem, ptx::smem_desc_sw128(a_addr + kATile + 32 * k), bdesc,
-                                      idesc, 1u);
+                    ptx::mma_bf16_ta(tmem, a_tm + 8 * k, bdesc, idesc, (i | k) != 0);
+                    if constexpr (SPLIT) ptx::mma_bf16_ta(tmem, a_tm + kACols + 8 * k, bdesc, idesc, 1u);
                 }
                 ptx::mma_commit(&ax_empty[s]);
             }
@@ -257,10 +263,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
     } else {
         // ---------------------------------------------------------------- dequant
-        // two threads per weight row: thread (row t, half h) writes 4 of the 8 16-byte
-        // chunks of each 64-k atom row (the chunks of 32-block 2j+h of atom j)
-        const int u = threadIdx.x - 64;
-        const int t = u & (kBN - 1), h = u >> 7;
+        // two threads per weight row: thread (row t, half h) produces 32 of the 64 bf16 of
+        // each 64-k step (32-block 2j+h of step j) and stores them into its TMEM lane t,
+        // 16 columns; a warp reaches only its lane quarter (warp % 4), so t = 32*(warp%4) + lane
+        const int t = 32 * (warp & 3) + lane, h = (warp - 2) >> 2;
+        const uint32_t a_lane = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t(kAccCols + 16 * h);
         const unsigned full = 0xffffffffu;
         bool ok = true;
         for (int r = 0; r < nr && ok; ++r) {
@@ -287,25 +294,29 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     ok = __all_sync(full, ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
                                                          p.status, kWaitLimitNs));
                     if (!ok) break;
+                    ptx::tc_fence_after();  // the MMAs that read this A stage have completed
                 }
-                uint8_t* arow = a_ring + s * kAT * kATile + t * 128;
-                const int sx = t & 7;  // 128B swizzle: 16-byte chunk c of row t lives at c ^ (t & 7)
+                const uint32_t a_dst = a_lane + uint32_t(s * kAT * kACols);
+                const int sx = t & 7;  // raw codes: 16-byte chunk c of row t lives at c ^ (t & 7)
+                uint32_t va[16], vl[16];  // this thread's 16 columns of the hi (and lo) tile
                 if constexpr (FMT == EMB_Q8_0) {
                     // atom j: codes 64j..64j+63 of the raw stage = plane j/2, chunks 4(j%2)..+3;
                     // this half: chunks 4(j%2)+2h, +1 (block 2j+h) -> output chunks 4h..4h+3
 #pragma unroll
-                    for (int cc = 2 * h; cc < 2 * h + 2; ++cc) {
+                    for (int e = 0; e < 2; ++e) {
+                        const int cc = 2 * h + e;
                         const int c = (j & 1) * 4 + cc;
                         const uint4 v = lds128(rbase + (j >> 1) * kPlane + ((c ^ sx) << 4));
                         uint4 h0, l0, h1, l1;
                         make_chunk<SPLIT>(v.x ^ 0x80808080u, v.y ^ 0x80808080u, d[j], nbd[j], h0, l0);
                         make_chunk<SPLIT>(v.z ^ 0x80808080u, v.w ^ 0x80808080u, d[j], nbd[j], h1, l1);
-                        const int o0 = 2 * cc, o1 = 2 * cc + 1;
-                        sts128(arow + ((o0 ^ sx) << 4), h0);
-                        sts128(arow + ((o1 ^ sx) << 4), h1);
+                        // output chunks 2cc, 2cc+1 (k = 16cc .. 16cc+15) -> columns 8e .. 8e+7
+                        const int q = 8 * e;
+                        va[q + 0] = h0.x; va[q + 1] = h0.y; va[q + 2] = h0.z; va[q + 3] = h0.w;
+                        va[q + 4] = h1.x; va[q + 5] = h1.y; va[q + 6] = h1.z; va[q + 7] = h1.w;
                         if constexpr (SPLIT) {
-                            sts128(arow + kATile + ((o0 ^ sx) << 4), l0);
-                            sts128(arow + kATile + ((o1 ^ sx) << 4), l1);
+                            vl[q + 0] = l0.x; vl[q + 1] = l0.y; vl[q + 2] = l0.z; vl[q + 3] = l0.w;
+                            vl[q + 4] = l1.x; vl[q + 5] = l1.y; vl[q + 6] = l1.z; vl[q + 7] = l1.w;
                         }
                     }
                 } else {
@@ -320,13 +331,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     make_chunk<SPLIT>((v.x >> 4) & m, (v.y >> 4) & m, d[j], nbd[j], hh[2], ll[2]); // 16..23
                     make_chunk<SPLIT>((v.z >> 4) & m, (v.w >> 4) & m, d[j], nbd[j], hh[3], ll[3]); // 24..31
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int o = 4 * h + q;
-                        sts128(arow + ((o ^ sx) << 4), hh[q]);
-                        if constexpr (SPLIT) sts128(arow + kATile + ((o ^ sx) << 4), ll[q]);
+                    for (int q = 0; q < 4; ++q) {  // output chunk 4h+q -> columns 4q .. 4q+3
+                        va[4 * q + 0] = hh[q].x; va[4 * q + 1] = hh[q].y;
+                        va[4 * q + 2] = hh[q].z; va[4 * q + 3] = hh[q].w;
+                        if constexpr (SPLIT) {
+                            vl[4 * q + 0] = ll[q].x; vl[4 * q + 1] = ll[q].y;
+                            vl[4 * q + 2] = ll[q].z; vl[4 * q + 3] = ll[q].w;
+                        }
                     }
                 }
-                ptx::fence_proxy_async_smem();
+                ptx::tmem_st_16(a_dst, va);
+                if constexpr (SPLIT) ptx::tmem_st_16(a_dst + kACols, vl);
+                ptx::tmem_st_wait();
+                ptx::tc_fence_before();  // the stores are ordered before the arrive
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(&a_full[s]);
             }
@@ -453,15 +470,23 @@ bool encode_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_
 
 constexpr int kSmemLimit = 227 * 1024;
 
-template <int FMT, bool SPLIT>
-int smem_bytes(int T, int S) {
-    return 1024 + S * ((SPLIT ? 2 : 1) * kATile + T * 128) +
-           kRawStages * (RawTraits<FMT>::bytes + kScaleTile) + (2 * kRawStages + 3 * S + 1) * 8 + 16;
-}
+// Every CTA allocates all 512 TMEM columns, so no two may share an SM (a second one
+// would block in tcgen05.alloc, and inside a split-K cluster wait on the first forever):
+// the dynamic shared memory is padded above half of the SM's.
+constexpr int kOneCtaPerSm = 120 * 1024;
 
 template <int FMT, bool SPLIT>
+int smem_bytes(int T, int S) {
+    const int need = 1024 + S * T * 128 + kRawStages * (RawTraits<FMT>::bytes + kScaleTile) +
+                     (2 * kRawStages + 3 * S + 1) * 8 + 16;
+    return need > kOneCtaPerSm ? need : kOneCtaPerSm;
+}
+
+// Ring depth: as many X stages as shared memory holds, at most as many A stages as fit
+// in TMEM beside the accumulator (8 single tiles or 4 hi/lo pairs).
+template <int FMT, bool SPLIT>
 int pick_stages(int T) {
-    int S = 6;
+    int S = (int(kTmemCols) - kAccCols) / ((SPLIT ? 2 : 1) * kACols);
     while (S > 2 && smem_bytes<FMT, SPLIT>(T, S) > kSmemLimit) --S;
     return S;
 }
@@ -517,7 +542,7 @@ cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl,
 int pick_splits(int64_t tiles, int T, int64_t K, int stages, bool split_operand) {
     const int64_t nr = (K + kKR - 1) / kKR;
     const double work_us = 2.0 * kBN * T * double(K) / 11.6e12 * 1e6 * (split_operand ? 2 : 1);
-    const int64_t ring = int64_t(stages) * ((split_operand ? 2 : 1) * kATile + int64_t(T) * 128);
+    const int64_t ring = int64_t(stages) * int64_t(T) * 128;
     const int64_t part = int64_t(kBN) * T * 4;
     int best = 1;
     double best_t = 1e30;
@@ -574,9 +599,7 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.T = T;
     p.stages = S;
     p.splits = pick_splits(int64_t(t_tiles) * tiles, T, g.K, S, split);
-    uint32_t cols = 32;
-    while (cols < uint32_t(T)) cols <<= 1;
-    p.tmem_cols = cols;
+    p.tmem_cols = kTmemCols;
     p.status = status;
     const int grid_x = int(t_tiles);
     if (g.fmt == EMB_Q8_0)
