@@ -15,11 +15,13 @@
 // by TMA, read by the MMA), which bound this kernel (measured on GB300: 100 -> 70 KB of
 // shared-memory traffic per 64-k step; M = 816 prefill 683 -> 736 TFLOP/s).
 //
-// Roles (320 threads):
+// Roles (352 threads):
 //   warp 0 lane 0 : TMA producer. Raw stages (256 codes of 128 rows + their 8 scales)
 //                   are fetched before griddepcontrol.wait (weights never depend on
 //                   the previous launch); X tiles (64 k x T tokens) after it.
 //   warp 1        : TMEM allocation; lane 0 issues the MMAs (4 x K=16 per 64-k stage).
+//                   It never waits on an mbarrier while MMAs are in flight: warp 10
+//                   waits for each stage and releases it through a named barrier.
 //   warps 2..9    : dequantisation (two threads per weight row, tcgen05.st into the
 //                   warp's lane quarter), then the epilogue.
 // Grid: x = token tile (fastest: CTAs sharing a weight tile run together), y = weight-row
@@ -48,7 +50,8 @@ constexpr int kKR = 256;                   // k per raw stage
 constexpr int kStepsPerRaw = kKR / kKC;    // 4
 constexpr int kRawStages = 2;
 constexpr int kDeqWarps = 8;               // dequantisation (then epilogue) warps
-constexpr int kThreads = 64 + 32 * kDeqWarps;
+constexpr int kWaitWarp = 2 + kDeqWarps;   // waits on the MMA warp's behalf (see the kernel)
+constexpr int kThreads = 32 * (kWaitWarp + 1);
 constexpr int kAccCols = 256;              // TMEM columns [0, 256): the fp32 accumulator (T <= 256)
 constexpr int kACols = kKC / 2;            // TMEM columns of one bf16 A tile (two values per column)
 constexpr uint32_t kTmemCols = 512;        // accumulator + A stages
@@ -81,6 +84,11 @@ struct RawTraits {
 
 __device__ __forceinline__ uint4 lds128(const uint8_t* p) {
     return *reinterpret_cast<const uint4*>(p);
+}
+
+// bar.sync on a named barrier with `count` threads (whole warps).
+__device__ __forceinline__ void named_sync(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
@@ -143,6 +151,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint64_t* acc_full = ax_empty + S;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    volatile int* mma_stop = abort_flag + 1;  // set by the waiter warp when a wait gave up
     // split-K partial tile [T][128] fp32 (token-major): reuses the X ring once every MMA
     // has completed
     float* part = reinterpret_cast<float*>(x_ring);
@@ -176,6 +185,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         ptx::mbar_init(acc_full, 1);
         *abort_flag = 0;
+        *mma_stop = 0;
         ptx::fence_mbar_init();
         ptx::prefetch_tmap(&p.x_map);
         ptx::prefetch_tmap(&p.codes_map[g]);
@@ -238,15 +248,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 ptx::mbar_wait(&x_full[i % S], (i / S) & 1, nullptr, p.status, kWaitLimitNs);
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            // ------------------------------------------------------------ MMA issuer
-            const uint32_t idesc = ptx::idesc_bf16_f32(kBN, T);
-            const uint32_t x0 = ptx::smem_u32(x_ring);
-            for (int i = 0; i < nk; ++i) {
+        // ---------------------------------------------------------------- MMA issuer
+        // Step i is released by the waiter warp through named barrier 1; this warp itself
+        // runs no mbarrier wait while MMAs are in flight (see kWaitWarp below).
+        const uint32_t idesc = ptx::idesc_bf16_f32(kBN, T);
+        const uint32_t x0 = ptx::smem_u32(x_ring);
+        for (int i = 0; i < nk; ++i) {
+            named_sync(1, 64);
+            if (*mma_stop) break;
+            if (lane == 0) {
                 const int s = i % S;
-                const uint32_t ph = (i / S) & 1;
-                if (!ptx::mbar_wait(&x_full[s], ph, abort_flag, p.status, kWaitLimitNs)) break;
-                if (!ptx::mbar_wait(&a_full[s], ph, abort_flag, p.status, kWaitLimitNs)) break;
                 ptx::tc_fence_after();
                 const uint32_t a_tm = tmem + uint32_t(kAccCols + s * kAT * kACols);
                 const uint32_t x_addr = x0 + s * T * 128;
@@ -258,10 +269,31 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 }
                 ptx::mma_commit(&ax_empty[s]);
             }
+            __syncwarp();
+        }
+        if (lane == 0) {
             ptx::mma_commit(acc_full);  // completes once every issued MMA has finished
             ptx::mbar_wait(acc_full, 0, nullptr, p.status, kWaitLimitNs);
         }
-    } else {
+    } else if (warp == kWaitWarp) {
+        // ---------------------------------------------------------------- waiter
+        // An mbarrier wait executed by the warp that issues tcgen05 MMAs is ordered behind
+        // that warp's in-flight MMAs, which drains the tensor pipe at every step (measured
+        // on GB300: 104 -> 330+ cycles per 128x208x16 MMA). This warp waits for step i's
+        // X tile and A tile and then releases the MMA warp through named barrier 1.
+        for (int i = 0; i < nk; ++i) {
+            const int s = i % S;
+            const uint32_t ph = (i / S) & 1;
+            if (lane == 0) {
+                const bool ok = ptx::mbar_wait(&x_full[s], ph, abort_flag, p.status, kWaitLimitNs) &&
+                                ptx::mbar_wait(&a_full[s], ph, abort_flag, p.status, kWaitLimitNs);
+                if (!ok) *mma_stop = 1;
+            }
+            __syncwarp();
+            named_sync(1, 64);
+            if (*mma_stop) break;
+        }
+    } else if (warp < 2 + kDeqWarps) {
         // ---------------------------------------------------------------- dequant
         // two threads per weight row: thread (row t, half h) produces 32 of the 64 bf16 of
         // each 64-k step (32-block 2j+h of step j) and stores them into its TMEM lane t,
