@@ -302,6 +302,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         const uint32_t a_lane = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t(kAccCols + 16 * h);
         const unsigned full = 0xffffffffu;
         bool ok = true;
+        // Software pipeline: step i's TMEM stores are completed (tcgen05.wait::st) and
+        // signalled only after step i+1 has been computed, so the store latency overlaps
+        // the next step's arithmetic instead of stalling this warp every step.
+        int pending = -1;  // A stage whose stores are in flight, not yet signalled
+        auto signal_pending = [&]() {
+            if (pending >= 0) {
+                ptx::tmem_st_wait();
+                ptx::tc_fence_before();  // the stores are ordered before the arrive
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&a_full[pending]);
+                pending = -1;
+            }
+        };
         for (int r = 0; r < nr && ok; ++r) {
             const int rs = r % kRawStages;
             ok = __all_sync(full, ptx::mbar_wait(&raw_full[rs], (r / kRawStages) & 1, abort_flag,
@@ -322,12 +335,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 const int i = r * kStepsPerRaw + j;
                 if (i >= nk) break;
                 const int s = i % S;
-                if (i >= S) {
-                    ok = __all_sync(full, ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
-                                                         p.status, kWaitLimitNs));
-                    if (!ok) break;
-                    ptx::tc_fence_after();  // the MMAs that read this A stage have completed
-                }
                 const uint32_t a_dst = a_lane + uint32_t(s * kAT * kACols);
                 const int sx = t & 7;  // raw codes: 16-byte chunk c of row t lives at c ^ (t & 7)
                 uint32_t va[16], vl[16];  // this thread's 16 columns of the hi (and lo) tile
@@ -372,17 +379,23 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         }
                     }
                 }
+                signal_pending();
+                if (i >= S) {
+                    ok = __all_sync(full, ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
+                                                         p.status, kWaitLimitNs));
+                    if (!ok) break;
+                    ptx::tc_fence_after();  // the MMAs that read this A stage have completed
+                }
                 ptx::tmem_st_16(a_dst, va);
                 if constexpr (SPLIT) ptx::tmem_st_16(a_dst + kACols, vl);
-                ptx::tmem_st_wait();
-                ptx::tc_fence_before();  // the stores are ordered before the arrive
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(&a_full[s]);
+                pending = s;
             }
             if (!ok) break;
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&raw_empty[rs]);
         }
+        if (ok) signal_pending();
+        ptx::tmem_st_wait();  // no store of this warp is left in flight, whatever happened
 
         // ---------------------------------------------------------------- epilogue
         ptx::griddep_wait();  // Y may be read or written by the previous launch
