@@ -134,3 +134,40 @@ def test_staged_gemv_fused_group(cuda_device, fmt):
     for (f, img, N, _, _, Y), W in zip(specs, host):
         Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
         check_close(Y.cpu().numpy(), Yref, B, f"fused staged N={N}")
+
+
+# Problems with at least 152 output tiles (128 weight rows x up to 256 tokens): several
+# waves of CTAs, tiles that straddle a ragged N, M and K (partial 64-k step and partial
+# 256-k raw stage), and a fused pair. Checked element by element against the oracle.
+MANY_TILE_SHAPES = [(208, 19461, 1056), (417, 6531, 2080), (816, 4864, 1024), (280, 11008, 1024)]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("M,N,K", MANY_TILE_SHAPES)
+def test_many_tile_gemm_parity(cuda_device, fmt, M, N, K):
+    Y, Yref, B, _, _ = run_case(fmt, M, N, K, seed=M * 3 + N + K)
+    check_close(Y, Yref, B, f"many-tile gemm fmt={fmt} M={M} N={N} K={K}")
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_many_tile_gemm_fused_pair_and_determinism(cuda_device, fmt):
+    M, K, Ns = 300, 1024, (9800, 9741)
+    Xb = activation_bits_np(M, K, 61)
+    X = to_dev_bf16(Xb)
+    specs, host = [], []
+    for i, N in enumerate(Ns):
+        W = weight_np(N, K, 62 + i)
+        img = emb.quantize(fmt, torch.from_numpy(W).cuda())
+        Y = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+        specs.append((fmt, img, N, K, X, Y))
+        host.append(W)
+    emb.emb_qlayer_seq(specs, M)
+    torch.cuda.synchronize()
+    first = [sp[5].clone() for sp in specs]
+    emb.emb_qlayer_seq(specs, M)
+    torch.cuda.synchronize()
+    for a, sp in zip(first, specs):
+        assert torch.equal(a.view(torch.int32), sp[5].view(torch.int32))
+    for (f, img, N, _, _, Y), W in zip(specs, host):
+        Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
+        check_close(Y.cpu().numpy(), Yref, B, f"fused many-tile N={N}")
