@@ -171,3 +171,40 @@ def test_many_tile_gemm_fused_pair_and_determinism(cuda_device, fmt):
     for (f, img, N, _, _, Y), W in zip(specs, host):
         Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
         check_close(Y.cpu().numpy(), Yref, B, f"fused many-tile N={N}")
+
+
+# 5..64 tokens with K >= 1024 (the action-chunk range): ragged token tails, ragged N, K
+# that is not a multiple of the 64-k step or the 256-k raw stage, and long rows.
+ACTION_CHUNK_SHAPES = [(5, 136, 1024), (8, 200, 1056), (9, 77, 2048), (16, 300, 1024), (17, 129, 1056),
+                   (33, 64, 4128), (50, 1000, 1024), (50, 130, 4096), (64, 257, 2080)]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("M,N,K", ACTION_CHUNK_SHAPES)
+def test_action_chunk_parity(cuda_device, fmt, M, N, K):
+    Y, Yref, B, _, _ = run_case(fmt, M, N, K, seed=M * 11 + N + K)
+    check_close(Y, Yref, B, f"action-chunk fmt={fmt} M={M} N={N} K={K}")
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_action_chunk_fused_group_and_determinism(cuda_device, fmt):
+    M, K, Ns = 50, 1024, (1024, 128, 128)
+    Xb = activation_bits_np(M, K, 71)
+    X = to_dev_bf16(Xb)
+    specs, host = [], []
+    for i, N in enumerate(Ns):
+        W = weight_np(N, K, 72 + i)
+        img = emb.quantize(fmt, torch.from_numpy(W).cuda())
+        Y = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+        specs.append((fmt, img, N, K, X, Y))
+        host.append(W)
+    emb.emb_qlayer_seq(specs, M)
+    torch.cuda.synchronize()
+    first = [sp[5].clone() for sp in specs]
+    emb.emb_qlayer_seq(specs, M)
+    torch.cuda.synchronize()
+    for a, sp in zip(first, specs):
+        assert torch.equal(a.view(torch.int32), sp[5].view(torch.int32))
+    for (f, img, N, _, _, Y), W in zip(specs, host):
+        Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
+        check_close(Y.cpu().numpy(), Yref, B, f"fused action-chunk N={N}")
