@@ -36,6 +36,8 @@
 // operand error from 2^-9 to 2^-17 relative (the 1e-3 * sum|w x| bound then holds for
 // every input, not only statistically).
 #include <cuda.h>
+#include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 
@@ -52,11 +54,12 @@ constexpr int kRawStages = 2;
 constexpr int kDeqWarps = 8;               // dequantisation (then epilogue) warps
 constexpr int kWaitWarp = 2 + kDeqWarps;   // waits on the MMA warp's behalf (see the kernel)
 constexpr int kThreads = 32 * (kWaitWarp + 1);
-constexpr int kAccCols = 256;              // TMEM columns [0, 256): the fp32 accumulator (T <= 256)
+constexpr int kAccCols = 256;              // TMEM columns [0, 256): one token tile's accumulator (T <= 256)
 constexpr int kACols = kKC / 2;            // TMEM columns of one bf16 A tile (two values per column)
 constexpr uint32_t kTmemCols = 512;        // accumulator + A stages
 constexpr int kPlane = kBN * 128;          // 16 KB: 128 rows x 128 bytes of codes
 constexpr int kScaleTile = kBN * 16;       // 2 KB: 128 rows x 8 fp16 scales
+constexpr int kMaxStages = 8;              // A/X ring depth, at most
 
 struct GemmParams {
     CUtensorMap x_map;                     // X [M][K] bf16, box {64, T}, 128B swizzle
@@ -67,9 +70,12 @@ struct GemmParams {
     int32_t tile0[kMaxGroup + 1];
     int32_t n_mats;
     int32_t M, K;
-    int32_t T;                             // tokens per CTA, multiple of 16, <= 256
+    int32_t T;                             // tokens per token tile, multiple of 16, <= 256
+    int32_t P;                             // token tiles per CTA (1, or 2 sharing each A tile)
     int32_t splits;                        // K splits (cluster size along z)
     int32_t stages;                        // A/X ring depth
+    int32_t a_gap0;                        // P = 2: TMEM column of the first A stage after tile 0's
+    int32_t a_per_gap;                     //   accumulator, and A stages per gap (see pick_stages_pair)
     uint32_t tmem_cols;
     int* status;
 };
@@ -131,16 +137,24 @@ __device__ __forceinline__ void make_chunk(uint32_t u0, uint32_t u1, float d, fl
     }
 }
 
-template <int FMT, bool SPLIT>
+// TMEM column of A stage s: after the accumulator (P = 1), or in the slots after each of
+// the two accumulators at columns 0 and 256 (P = 2).
+template <int P, bool SPLIT>
+__device__ __forceinline__ uint32_t a_stage_col(int s, int gap0, int per_gap) {
+    if constexpr (P == 1) return uint32_t(kAccCols + s * (SPLIT ? 2 : 1) * kACols);
+    return uint32_t(s < per_gap ? gap0 + s * kACols : kAccCols + gap0 + (s - per_gap) * kACols);
+}
+
+template <int FMT, bool SPLIT, int P>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmParams p) {
     using RT = RawTraits<FMT>;
-    constexpr int kAT = SPLIT ? 2 : 1;
+    static_assert(P == 1 || (P == 2 && !SPLIT), "two token tiles only without the split operand");
     extern __shared__ uint8_t smem_dyn[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
                                                ~uintptr_t(1023));
     const int S = p.stages, T = p.T;
-    uint8_t* x_ring = base;                                     // S x T x 128 B
-    uint8_t* r_ring = x_ring + S * T * 128;                     // 2 x RT::bytes
+    uint8_t* x_ring = base;                                     // S x P x T x 128 B
+    uint8_t* r_ring = x_ring + S * P * T * 128;                 // 2 x RT::bytes
     uint8_t* s_ring = r_ring + kRawStages * RT::bytes;          // 2 x 2 KB
     uint64_t* bars = reinterpret_cast<uint64_t*>(s_ring + kRawStages * kScaleTile);
     uint64_t* raw_full = bars;
@@ -163,7 +177,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     for (int i = 1; i < kMaxGroup; ++i)
         if (i < p.n_mats && tile >= p.tile0[i]) g = i;
     const int n0 = (tile - p.tile0[g]) * kBN;
-    const int m0 = blockIdx.x * T;
+    const int m0 = blockIdx.x * P * T;  // first token of the CTA's first token tile
     const int N = p.N[g], M = p.M, K = p.K;
     // this CTA's K range: split-K over raw stages of 256
     const int splits = gridDim.z, split = blockIdx.z;
@@ -235,9 +249,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 if (i >= S && !ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
                                               p.status, kWaitLimitNs))
                     break;
-                ptx::mbar_arrive_expect_tx(&x_full[s], uint32_t(T) * 128u);
-                ptx::tma_load_2d(x_ring + s * T * 128, &p.x_map, &x_full[s], (ks0 + i) * kKC, m0,
-                                 pol_x);
+                ptx::mbar_arrive_expect_tx(&x_full[s], uint32_t(P * T) * 128u);
+#pragma unroll
+                for (int q = 0; q < P; ++q)  // a tile past M reads zeros (its outputs are not stored)
+                    ptx::tma_load_2d(x_ring + (s * P + q) * T * 128, &p.x_map, &x_full[s],
+                                     (ks0 + i) * kKC, m0 + q * T, pol_x);
                 ++x_issued;
             }
             // every issued copy must land before this CTA's shared memory can be released
@@ -259,13 +275,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             if (lane == 0) {
                 const int s = i % S;
                 ptx::tc_fence_after();
-                const uint32_t a_tm = tmem + uint32_t(kAccCols + s * kAT * kACols);
-                const uint32_t x_addr = x0 + s * T * 128;
+                const uint32_t a_tm = tmem + a_stage_col<P, SPLIT>(s, p.a_gap0, p.a_per_gap);
 #pragma unroll
-                for (int k = 0; k < kKC / 16; ++k) {
-                    const uint64_t bdesc = ptx::smem_desc_sw128(x_addr + 32 * k);
-                    ptx::mma_bf16_ta(tmem, a_tm + 8 * k, bdesc, idesc, (i | k) != 0);
-                    if constexpr (SPLIT) ptx::mma_bf16_ta(tmem, a_tm + kACols + 8 * k, bdesc, idesc, 1u);
+                for (int q = 0; q < P; ++q) {
+                    // token tile q: its own X tile and accumulator, the same A tile
+                    const uint32_t x_addr = x0 + (s * P + q) * T * 128;
+                    const uint32_t d_tm = tmem + uint32_t(q * kAccCols);
+#pragma unroll
+                    for (int k = 0; k < kKC / 16; ++k) {
+                        const uint64_t bdesc = ptx::smem_desc_sw128(x_addr + 32 * k);
+                        ptx::mma_bf16_ta(d_tm, a_tm + 8 * k, bdesc, idesc, (i | k) != 0);
+                        if constexpr (SPLIT) ptx::mma_bf16_ta(d_tm, a_tm + kACols + 8 * k, bdesc, idesc, 1u);
+                    }
                 }
                 ptx::mma_commit(&ax_empty[s]);
             }
@@ -299,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         // each 64-k step (32-block 2j+h of step j) and stores them into its TMEM lane t,
         // 16 columns; a warp reaches only its lane quarter (warp % 4), so t = 32*(warp%4) + lane
         const int t = 32 * (warp & 3) + lane, h = (warp - 2) >> 2;
-        const uint32_t a_lane = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t(kAccCols + 16 * h);
+        const uint32_t a_lane = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t(16 * h);
         const unsigned full = 0xffffffffu;
         bool ok = true;
         // Software pipeline: step i's TMEM stores are completed (tcgen05.wait::st) and
@@ -335,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 const int i = r * kStepsPerRaw + j;
                 if (i >= nk) break;
                 const int s = i % S;
-                const uint32_t a_dst = a_lane + uint32_t(s * kAT * kACols);
+                const uint32_t a_dst = a_lane + a_stage_col<P, SPLIT>(s, p.a_gap0, p.a_per_gap);
                 const int sx = t & 7;  // raw codes: 16-byte chunk c of row t lives at c ^ (t & 7)
                 uint32_t va[16], vl[16];  // this thread's 16 columns of the hi (and lo) tile
                 if constexpr (FMT == EMB_Q8_0) {
@@ -402,13 +423,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         ok = __all_sync(full, ok && ptx::mbar_wait(acc_full, 0, abort_flag, p.status, kWaitLimitNs));
         if (ok) {
             ptx::tc_fence_after();
-            // warps 2..9: TMEM lane quarter = warp % 4; two warps per quarter split the columns
+            // warps 2..9: TMEM lane quarter = warp % 4; the two warps of a quarter split the
+            // columns of one token tile, or (P = 2) take one token tile each
             const int quarter = warp & 3, half = (warp - 2) >> 2;
             const int csplit = ((T >> 1) + 15) & ~15;
-            const int cbeg = half ? csplit : 0, cend = half ? T : min(csplit, T);
+            const int tt = (P == 2) ? half : 0;  // token tile read by this warp
+            const int cbeg = (P == 2 || !half) ? 0 : csplit;
+            const int cend = (P == 2 || half) ? T : min(csplit, T);
             const int row = quarter * 32 + lane;
-            const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16);
+            const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16) + uint32_t(tt * kAccCols);
             const int n = n0 + row;
+            const int mt = m0 + tt * T;  // first token of that tile
             float* Y = p.Y[g];
             for (int c0 = cbeg; c0 < cend; c0 += 16) {
                 uint32_t v[16];
@@ -418,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     if (n < N) {
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
-                            const int m = m0 + c0 + e;
+                            const int m = mt + c0 + e;
                             if (m < M) Y[int64_t(m) * N + n] = __uint_as_float(v[e]);
                         }
                     }
@@ -521,8 +546,8 @@ constexpr int kSmemLimit = 227 * 1024;
 constexpr int kOneCtaPerSm = 120 * 1024;
 
 template <int FMT, bool SPLIT>
-int smem_bytes(int T, int S) {
-    const int need = 1024 + S * T * 128 + kRawStages * (RawTraits<FMT>::bytes + kScaleTile) +
+int smem_bytes(int T, int S, int P) {
+    const int need = 1024 + S * P * T * 128 + kRawStages * (RawTraits<FMT>::bytes + kScaleTile) +
                      (2 * kRawStages + 3 * S + 1) * 8 + 16;
     return need > kOneCtaPerSm ? need : kOneCtaPerSm;
 }
@@ -532,15 +557,28 @@ int smem_bytes(int T, int S) {
 template <int FMT, bool SPLIT>
 int pick_stages(int T) {
     int S = (int(kTmemCols) - kAccCols) / ((SPLIT ? 2 : 1) * kACols);
-    while (S > 2 && smem_bytes<FMT, SPLIT>(T, S) > kSmemLimit) --S;
+    while (S > 2 && smem_bytes<FMT, SPLIT>(T, S, 1) > kSmemLimit) --S;
     return S;
 }
 
-template <int FMT, bool SPLIT>
+// Two token tiles per CTA (P = 2): the accumulators sit at TMEM columns 0 and 256 and the
+// A stages in the 32-column slots after each (so T <= 224). Returns the ring depth that
+// fits TMEM and shared memory (0 if fewer than two) and fills the stages' columns.
+template <int FMT>
+int pick_stages_pair(int T, int& gap0, int& per_gap) {
+    gap0 = int(roundup(T, 32));
+    per_gap = (kAccCols - gap0) / kACols;
+    int S = std::min(2 * per_gap, kMaxStages);
+    while (S > 2 && smem_bytes<FMT, false>(T, S, 2) > kSmemLimit) --S;
+    if (S < 2 || smem_bytes<FMT, false>(T, S, 2) > kSmemLimit) return 0;
+    return S;
+}
+
+template <int FMT, bool SPLIT, int P>
 cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl, cudaStream_t s) {
     // grid: x = token tile (fastest, so the CTAs sharing a weight tile run together and
     // read it from L2 after the first), y = weight-row tile, z = K split (one cluster)
-    const int bytes = smem_bytes<FMT, SPLIT>(p.T, p.stages);
+    const int bytes = smem_bytes<FMT, SPLIT>(p.T, p.stages, p.P);
     // the opt-in shared-memory size is a per-device function attribute
     static std::mutex mu;
     static bool done[64] = {};
@@ -550,7 +588,7 @@ cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl,
     {
         std::lock_guard<std::mutex> lock(mu);
         if (dev < 0 || dev >= 64 || !done[dev]) {
-            e = cudaFuncSetAttribute(gemm_tc_kernel<FMT, SPLIT>,
+            e = cudaFuncSetAttribute(gemm_tc_kernel<FMT, SPLIT, P>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
             if (e != cudaSuccess) return e;
             if (dev >= 0 && dev < 64) done[dev] = true;
@@ -577,7 +615,18 @@ cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl,
     }
     cfg.attrs = attr;
     cfg.numAttrs = na;
-    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<FMT, SPLIT>, p);
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<FMT, SPLIT, P>, p);
+}
+
+int sm_count() {
+    static std::mutex mu;
+    static int counts[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!counts[dev] && cudaDeviceGetAttribute(&counts[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        counts[dev] = 0;
+    return counts[dev];
 }
 
 // K splits (1, 2 or 4; one cluster of CTAs per output tile): the count minimising a
@@ -610,17 +659,53 @@ bool gemm_tc_supported(const GroupRef& g) {
 cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s) {
     GemmParams p;
     memset(&p, 0, sizeof(p));
-    // tokens per CTA: balanced tiles of at most 256, rounded up to the MMA's N granule (16)
+    int tiles = 0;
+    for (int i = 0; i < g.n_mats; ++i) tiles += int((g.mats[i].N + kBN - 1) / kBN);
+    // one token tile per CTA: balanced tiles of at most 256, rounded up to the MMA's N granule
     const int64_t t_tiles = (g.M + 255) / 256;
-    const int T = int(roundup((g.M + t_tiles - 1) / t_tiles, 16));
+    int T = int(roundup((g.M + t_tiles - 1) / t_tiles, 16));
     const bool split = g.K < 1024;
-    const int S = g.fmt == EMB_Q8_0 ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
-                                    : (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T));
+    int S = g.fmt == EMB_Q8_0 ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
+                              : (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T));
+    int splits = pick_splits(int64_t(t_tiles) * tiles, T, g.K, S, split);
+    int P = 1, grid_x = int(t_tiles);
+    // Two token tiles per CTA halve the dequantisation per token (each A tile feeds the MMAs
+    // of both). Time model in cycles, fitted to GB300 measurements of both formats: per
+    // 64-k step the larger of the dequantisation (~1050) and the MMA work (~5.2 per token
+    // of the CTA), plus ~3900 of pipeline fill and drain per CTA, times the waves of CTAs
+    // over the SMs. Pairs win where one tile per CTA is dequantisation-bound (T <= ~200)
+    // and the pairs do not add a wave: Llama-7B qkv at M = 280, 455 -> 678 TFLOP/s; gate/up
+    // 547 -> 610. At M = 816 (T = 208) one tile per CTA is already MMA-bound and pairs lose
+    // (847 -> 772); narrow layers keep one tile per CTA and split K instead.
+    if (!split && t_tiles >= 2) {
+        const int64_t t2 = 2 * ((g.M + 447) / 448);  // even count of tiles of at most 224
+        const int T2 = int(roundup((g.M + t2 - 1) / t2, 16));
+        int gap0 = 0, per_gap = 0;
+        const int S2 = (g.fmt == EMB_Q8_0) ? pick_stages_pair<EMB_Q8_0>(T2, gap0, per_gap)
+                                           : pick_stages_pair<EMB_Q4_0>(T2, gap0, per_gap);
+        const int sms = sm_count();
+        if (S2 >= 2 && T2 <= 224 && sms > 0) {
+            const double nk = double((g.K + kKC - 1) / kKC);
+            auto waves = [&](int64_t ctas) { return double((ctas + sms - 1) / sms); };
+            const double c1 = waves(int64_t(t_tiles) * tiles * splits) *
+                              (std::ceil(nk / splits) * std::max(1050.0, 5.2 * T) + 3900.0);
+            const double c2 = waves(int64_t(t2 / 2) * tiles) * (nk * std::max(1050.0, 5.2 * 2 * T2) + 3900.0);
+            if (c2 < 0.95 * c1) {
+                P = 2;
+                T = T2;
+                S = S2;
+                splits = 1;
+                grid_x = int(t2 / 2);
+                p.a_gap0 = gap0;
+                p.a_per_gap = per_gap;
+            }
+        }
+    }
     if (!encode_2d(&p.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.X, uint64_t(g.K), uint64_t(g.M),
                    uint64_t(g.K) * 2, kKC, uint32_t(T), CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B))
         return cudaErrorInvalidValue;
-    int tiles = 0;
+    tiles = 0;
     for (int i = 0; i < g.n_mats; ++i) {
         const MatRef& mr = g.mats[i];
         const uint64_t row_bytes = g.fmt == EMB_Q8_0 ? uint64_t(g.K) : uint64_t(g.K) / 2;
@@ -642,16 +727,18 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.M = int32_t(g.M);
     p.K = int32_t(g.K);
     p.T = T;
+    p.P = P;
     p.stages = S;
-    p.splits = pick_splits(int64_t(t_tiles) * tiles, T, g.K, S, split);
+    p.splits = splits;
     p.tmem_cols = kTmemCols;
     p.status = status;
-    const int grid_x = int(t_tiles);
     if (g.fmt == EMB_Q8_0)
-        return split ? launch_kernel<EMB_Q8_0, true>(p, grid_x, tiles, pdl, s)
-                     : launch_kernel<EMB_Q8_0, false>(p, grid_x, tiles, pdl, s);
-    return split ? launch_kernel<EMB_Q4_0, true>(p, grid_x, tiles, pdl, s)
-                 : launch_kernel<EMB_Q4_0, false>(p, grid_x, tiles, pdl, s);
+        return split    ? launch_kernel<EMB_Q8_0, true, 1>(p, grid_x, tiles, pdl, s)
+               : P == 2 ? launch_kernel<EMB_Q8_0, false, 2>(p, grid_x, tiles, pdl, s)
+                        : launch_kernel<EMB_Q8_0, false, 1>(p, grid_x, tiles, pdl, s);
+    return split    ? launch_kernel<EMB_Q4_0, true, 1>(p, grid_x, tiles, pdl, s)
+           : P == 2 ? launch_kernel<EMB_Q4_0, false, 2>(p, grid_x, tiles, pdl, s)
+                    : launch_kernel<EMB_Q4_0, false, 1>(p, grid_x, tiles, pdl, s);
 }
 
 }  // namespace emb

@@ -151,7 +151,7 @@ def test_many_tile_gemm_parity(cuda_device, fmt, M, N, K):
 
 @pytest.mark.parametrize("fmt", FMTS)
 def test_many_tile_gemm_fused_pair_and_determinism(cuda_device, fmt):
-    M, K, Ns = 300, 1024, (9800, 9741)
+    M, K, Ns = 280, 1024, (11008, 11001)   # two token tiles per CTA (as Llama-7B gate/up)
     Xb = activation_bits_np(M, K, 61)
     X = to_dev_bf16(Xb)
     specs, host = [], []
@@ -171,6 +171,20 @@ def test_many_tile_gemm_fused_pair_and_determinism(cuda_device, fmt):
     for (f, img, N, _, _, Y), W in zip(specs, host):
         Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
         check_close(Y.cpu().numpy(), Yref, B, f"fused many-tile N={N}")
+
+
+# Wide layers at 280..561 tokens where one CTA computes two token tiles from each
+# dequantised weight tile: several waves, ragged N, the last token tile partly past M
+# (420 = 2 x 224 - 28 with the widest pair tiles, 561 = 4 x 144 - 15), K not a multiple
+# of the 256-k raw stage.
+PAIR_SHAPES = [(420, 30000, 1024), (561, 19000, 1056), (300, 40000, 1024), (280, 23000, 2080)]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("M,N,K", PAIR_SHAPES)
+def test_token_pair_gemm_parity(cuda_device, fmt, M, N, K):
+    Y, Yref, B, _, _ = run_case(fmt, M, N, K, seed=M * 13 + N + K)
+    check_close(Y, Yref, B, f"token-pair gemm fmt={fmt} M={M} N={N} K={K}")
 
 
 # 5..64 tokens with K >= 1024 (the action-chunk range): ragged token tails, ragged N, K
