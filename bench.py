@@ -172,23 +172,40 @@ WORKLOADS = {
 
 
 def build_chain(w: wl.Workload, device):
-    """Device weights (generated, quantised, fp32 freed), activations and outputs."""
+    """Device weights (generated, quantised, fp32 freed), activations and outputs. All
+    activations of the chain live in one device arena and all outputs in another (views
+    at 256-byte offsets), so a step moves them with one copy each way."""
     import torch
     import paper_2607_02501_gb300 as emb
+
+    def r256(n):
+        return (n + 255) // 256 * 256
+    x_bytes = sum(r256(w.M * g[0].K * 2) for g in w.groups)
+    y_bytes = sum(r256(w.M * lin.N * 4) for g in w.groups for lin in g)
+    x_arena = torch.empty(x_bytes, dtype=torch.uint8, device=device)
+    y_arena = torch.empty(y_bytes, dtype=torch.uint8, device=device)
     specs, xs, ys = [], [], []
+    xo = yo = 0
     for group in w.groups:
         K = group[0].K
-        X = wl.activation_torch(w.M, K, wl.activation_seed(group[0]), device=device)
+        X = x_arena[xo:xo + w.M * K * 2].view(torch.bfloat16).view(w.M, K)
+        X.copy_(wl.activation_torch(w.M, K, wl.activation_seed(group[0]), device=device))
+        xo += r256(w.M * K * 2)
         xs.append(X)
         for lin in group:
             W = wl.weight_torch(lin, device=device)
             img = emb.quantize(w.fmt, W)
             del W
-            Y = torch.empty(w.M, lin.N, dtype=torch.float32, device=device)
+            Y = y_arena[yo:yo + w.M * lin.N * 4].view(torch.float32).view(w.M, lin.N)
+            yo += r256(w.M * lin.N * 4)
             ys.append(Y)
             specs.append((w.fmt, img, lin.N, lin.K, X, Y))
     torch.cuda.synchronize()
+    build_chain.arenas[id(specs)] = (x_arena, y_arena)
     return specs, xs, ys
+
+
+build_chain.arenas = {}   # id(specs) -> (activation arena, output arena)
 
 
 def count_launches(specs) -> int:
@@ -206,19 +223,15 @@ def count_launches(specs) -> int:
 
 
 def capture_graph(specs, M):
+    """The chain recorded by the library (emb_chain_create) after one eager call (module
+    load); returns an object whose replay() launches the whole chain with one call."""
     import torch
     import paper_2607_02501_gb300 as emb
-    layers = emb.make_layers(specs)
-    s = torch.cuda.Stream()
-    s.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(s):
-        emb.emb_qlayer_seq(layers, M)      # first call: module load, tensor-map setup
+    emb.emb_qlayer_seq(specs, M)
     torch.cuda.synchronize()
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=s):
-        emb.emb_qlayer_seq(layers, M)
-    torch.cuda.synchronize()
-    return g, layers
+    rec = emb.RecordedChain(specs, M)
+    rec.replay = rec.launch
+    return rec, rec.layers
 
 
 # ------------------------------------------------------------------ CPU oracle timing
@@ -473,20 +486,21 @@ def measure_e2e(chains, args, dev, dist, tensor_bound):
     output back, synchronise."""
     import torch
     import paper_2607_02501_gb300 as emb
-    host_x = [[x.cpu().pin_memory() for x in c["xs"]] for c in chains]
-    host_y = [[torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in c["ys"]] for c in chains]
-    h2d = sum(x.numel() * x.element_size() for hx in host_x for x in hx)
-    d2h = sum(y.numel() * y.element_size() for hy in host_y for y in hy)
+    arenas = [build_chain.arenas[id(c["specs"])] for c in chains]
+    host_x = [xa.cpu().pin_memory() for xa, _ in arenas]
+    host_y = [torch.empty(ya.shape, dtype=ya.dtype).pin_memory() for _, ya in arenas]
+    h2d = sum(x.numel() * x.element_size() for x in host_x)   # the bytes each step copies
+    d2h = sum(y.numel() * y.element_size() for y in host_y)
     steps = max(1, min(args.steps, 200))
 
     def one_step():
+        # per chain: every activation in (one copy of the arena), the recorded chain
+        # (one call), every output back (one copy)
         for k, c in enumerate(chains):
-            for hx, x in zip(host_x[k], c["xs"]):
-                x.copy_(hx, non_blocking=True)
+            arenas[k][0].copy_(host_x[k], non_blocking=True)
             for _ in range(c["w"].repeats):
-                emb.emb_qlayer_seq(c["layers"], c["w"].M)
-            for hy, y in zip(host_y[k], c["ys"]):
-                hy.copy_(y, non_blocking=True)
+                c["graph"].replay()
+            host_y[k].copy_(arenas[k][1], non_blocking=True)
         torch.cuda.synchronize()
 
     for _ in range(3):
@@ -505,7 +519,8 @@ def measure_e2e(chains, args, dev, dist, tensor_bound):
         val, unit = world * work * steps / el / 1e9, "GB/s"
     return {"value": val, "unit": unit, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "steps": steps, "ms_per_step": el / steps * 1e3,
-            "how": "eager emb_qlayer_seq per format + pinned H2D of X / D2H of Y each step"}
+            "how": "per format: one pinned H2D copy of all activations, one emb_chain_launch "
+                   "of the recorded chain, one D2H copy of all outputs; synchronise each step"}
 
 
 def main(argv=None):

@@ -21,9 +21,10 @@
  *     layout), X is [M][K] row-major bf16 (passed as its 16-bit patterns),
  *     Y is [M][N] row-major fp32, and Y[m][n] = sum_k w'[n][k] * x[m][k].
  *   - Every pointer argument is DEVICE memory owned by the caller, except the
- *     `layers` array of emb_qlayer_seq, which is host memory read during the
- *     call only. The library allocates nothing and keeps no per-call state; all
- *     calls are reentrant and thread-safe.
+ *     `layers` arrays of emb_qlayer_seq / emb_chain_create, which are host memory
+ *     read during the call only. The library allocates no device memory and keeps
+ *     no per-call state (a recorded chain is a caller-owned handle); all calls are
+ *     reentrant and thread-safe.
  *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
  *     stream) without any host synchronisation, except emb_device_status.
  *   - Argument errors are reported BEFORE anything is enqueued. Launch errors
@@ -143,6 +144,32 @@ EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, 
  * bytes (may be NULL when that is 0). */
 EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M,
                           void* workspace, size_t ws_bytes, emb_stream_t stream);
+
+/* ------------------------------------------------------------ recorded chains
+ * The paper's "graph replay" and "buffer reuse" (Section 3.2, design principle 2): the
+ * launches that emb_qlayer_seq(layers, n_layers, M, workspace, ws_bytes, ...) enqueues
+ * are recorded once into a CUDA graph and then replayed with one call, so a closed-loop
+ * step costs one host call instead of one per launch group. */
+typedef struct emb_chain_st* emb_chain_t;
+
+/* Record the chain. Arguments, validation and error codes are those of emb_qlayer_seq
+ * (nothing is launched: the launches are captured on a private stream of the current
+ * device). The recording holds the layers' pointers: every replay reads the X buffers
+ * and fully overwrites the Y buffers given here, so callers refill the X buffers between
+ * replays and keep every buffer (and the workspace) alive until emb_chain_destroy.
+ * Results of a replay are bitwise those of emb_qlayer_seq on the same inputs.
+ * On success *chain receives a handle owned by the caller; on failure it is NULL.
+ * Errors: EMB_EINVAL (also for a NULL chain pointer), EMB_EALIGN, EMB_EUNSUPPORTED,
+ * EMB_ECUDA (stream capture or graph instantiation failed). */
+EMB_API emb_status emb_chain_create(const emb_qlayer* layers, int n_layers, int64_t M,
+                            void* workspace, size_t ws_bytes, emb_chain_t* chain);
+
+/* Enqueue one replay of the recorded chain on `stream` (a stream of the device it was
+ * recorded on). EMB_EINVAL for a NULL handle, EMB_ECUDA if the launch fails. */
+EMB_API emb_status emb_chain_launch(emb_chain_t chain, emb_stream_t stream);
+
+/* Free the recording (NULL is a no-op). Replays already enqueued still complete. */
+EMB_API emb_status emb_chain_destroy(emb_chain_t chain);
 
 /* ---------------------------------------------------------------- test support
  * Dequantise W_blocks to fp32 [N][K] (w' exactly: the products are exact in fp32). */

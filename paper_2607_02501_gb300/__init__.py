@@ -78,6 +78,12 @@ def lib():
     L.emb_qlayer_seq_workspace.restype = sz
     L.emb_qlayer_seq.argtypes = [ctypes.POINTER(emb_qlayer), i32, i64, vp, sz, vp]
     L.emb_qlayer_seq.restype = i32
+    L.emb_chain_create.argtypes = [ctypes.POINTER(emb_qlayer), i32, i64, vp, sz, ctypes.POINTER(vp)]
+    L.emb_chain_create.restype = i32
+    L.emb_chain_launch.argtypes = [vp, vp]
+    L.emb_chain_launch.restype = i32
+    L.emb_chain_destroy.argtypes = [vp]
+    L.emb_chain_destroy.restype = i32
     for name in ("emb_dequantize_f32", "emb_dequantize_bf16"):
         getattr(L, name).argtypes = [i32, vp, i64, i64, vp, vp]
         getattr(L, name).restype = i32
@@ -165,6 +171,49 @@ def emb_qlayer_seq(layers, M: int, workspace=None, ws_bytes: int = 0, stream=Non
     arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
     _check(lib().emb_qlayer_seq(arr, len(arr), M, _ptr(workspace), ws_bytes, _stream(stream)),
            "emb_qlayer_seq")
+
+
+def emb_chain_create(layers, M: int, workspace=None, ws_bytes: int = 0) -> int:
+    """Record a chain; returns the handle (an address). See RecordedChain for a wrapper
+    that also keeps the layers' tensors alive."""
+    arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
+    h = ctypes.c_void_p()
+    _check(lib().emb_chain_create(arr, len(arr), M, _ptr(workspace), ws_bytes, ctypes.byref(h)),
+           "emb_chain_create")
+    return int(h.value)
+
+
+def emb_chain_launch(chain: int, stream=None) -> None:
+    _check(lib().emb_chain_launch(chain, _stream(stream)), "emb_chain_launch")
+
+
+def emb_chain_destroy(chain: int) -> None:
+    _check(lib().emb_chain_destroy(chain), "emb_chain_destroy")
+
+
+class RecordedChain:
+    """emb_qlayer_seq recorded once (emb_chain_create) and replayed with one call per
+    step. Holds the specs so that every buffer the recording points at stays alive."""
+
+    def __init__(self, specs, M: int):
+        self.specs = list(specs)
+        self.layers = make_layers(self.specs)
+        self.M = M
+        self.handle = emb_chain_create(self.layers, M)
+
+    def launch(self, stream=None) -> None:
+        emb_chain_launch(self.handle, stream)
+
+    def close(self) -> None:
+        if self.handle:
+            emb_chain_destroy(self.handle)
+            self.handle = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def emb_dequantize_f32(fmt: int, W_blocks, N: int, K: int, out, stream=None) -> None:

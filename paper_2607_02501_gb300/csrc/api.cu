@@ -204,14 +204,13 @@ size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t 
     return 0;
 }
 
-emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
-                          size_t ws_bytes, emb_stream_t stream) {
-    (void)workspace;
-    (void)ws_bytes;
+// Validation of one chain and its launch groups (nothing enqueued).
+static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
+                              std::vector<GroupRef>& refs) {
     const emb_status st = check_seq(layers, n_layers, M);
     if (st != EMB_OK) return st;
     const auto groups = plan_groups(layers, n_layers, M);
-    std::vector<GroupRef> refs;
+    refs.clear();
     refs.reserve(groups.size());
     for (const auto& gr : groups) {
         const emb_qlayer& L0 = layers[gr.first];
@@ -229,7 +228,10 @@ emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, voi
         if (M > kGemvMaxM && !gemm_tc_supported(g)) return EMB_EUNSUPPORTED;
         refs.push_back(g);
     }
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    return EMB_OK;
+}
+
+static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s) {
     for (size_t i = 0; i < refs.size(); ++i) {
         // the first launch must not overlap whatever the caller enqueued before (it may
         // have produced the weights); later ones overlap their weight fetch with the
@@ -238,6 +240,71 @@ emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, voi
         if (e != cudaSuccess) return EMB_ECUDA;
     }
     return EMB_OK;
+}
+
+emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
+                          size_t ws_bytes, emb_stream_t stream) {
+    (void)workspace;
+    (void)ws_bytes;
+    std::vector<GroupRef> refs;
+    const emb_status st = prepare_seq(layers, n_layers, M, refs);
+    if (st != EMB_OK) return st;
+    return enqueue_seq(refs, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"
+
+// A recorded chain: the executable CUDA graph of one emb_qlayer_seq call.
+struct emb_chain_st {
+    cudaGraphExec_t exec;
+};
+
+extern "C" {
+
+emb_status emb_chain_create(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
+                            size_t ws_bytes, emb_chain_t* chain) {
+    (void)workspace;
+    (void)ws_bytes;
+    if (!chain) return EMB_EINVAL;
+    *chain = nullptr;
+    std::vector<GroupRef> refs;
+    emb_status st = prepare_seq(layers, n_layers, M, refs);
+    if (st != EMB_OK) return st;
+    // capture the chain's launches on a private stream (thread-local capture mode, so other
+    // threads' CUDA calls are unaffected), then instantiate the graph once
+    cudaStream_t s = nullptr;
+    if (cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) != cudaSuccess) return EMB_ECUDA;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+        cudaStreamDestroy(s);
+        return EMB_ECUDA;
+    }
+    st = enqueue_seq(refs, s);
+    const cudaError_t ec = cudaStreamEndCapture(s, &graph);  // ends the capture in every case
+    if (st == EMB_OK && ec != cudaSuccess) st = EMB_ECUDA;
+    if (st == EMB_OK && cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) st = EMB_ECUDA;
+    if (graph) cudaGraphDestroy(graph);
+    cudaStreamDestroy(s);
+    if (st != EMB_OK) {
+        if (exec) cudaGraphExecDestroy(exec);
+        return st;
+    }
+    *chain = new emb_chain_st{exec};
+    return EMB_OK;
+}
+
+emb_status emb_chain_launch(emb_chain_t chain, emb_stream_t stream) {
+    if (!chain) return EMB_EINVAL;
+    return from_cuda(cudaGraphLaunch(chain->exec, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+emb_status emb_chain_destroy(emb_chain_t chain) {
+    if (!chain) return EMB_OK;
+    // an executable graph that is still running is freed once it completes
+    const cudaError_t e = cudaGraphExecDestroy(chain->exec);
+    delete chain;
+    return from_cuda(e);
 }
 
 emb_status emb_dequantize_f32(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
@@ -287,8 +354,9 @@ const char* emb_status_string(emb_status status) {
 }
 
 const char* emb_build_info(void) {
-    return "libembqmm: sm_103a; Q8_0/Q4_0; GEMV (M<=4, register dequant, FFMA2) + "
-           "tcgen05 GEMM (M>4, TMA + smem dequant to bf16, TMEM accumulators)";
+    return "libembqmm: sm_103a; Q8_0/Q4_0; GEMV (M<=4: staged/register FFMA2, Q4_0 mma.sync at M>=2) + "
+           "tcgen05 GEMM (M>4: TMA, dequant to bf16 A tiles in TMEM, TMEM accumulators); "
+           "recorded chains (CUDA graphs)";
 }
 
 }  // extern "C"

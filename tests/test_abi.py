@@ -17,7 +17,7 @@ def L():
 
 def test_every_declared_symbol_is_exported(L):
     names = emb.declared_symbols()
-    assert len(names) == 12
+    assert len(names) == 15
     for n in names:
         assert hasattr(L, n), n
 
@@ -126,6 +126,24 @@ def test_seq_workspace_is_zero_for_valid_chains(L):
     chain = _layers([(0, A, 128, 64, B, C), (1, A + (64 << 20), 256, 64, B, C + (1 << 20))])
     assert emb.emb_qlayer_seq_workspace(chain, 1) == 0
     assert emb.emb_qlayer_seq_workspace(chain, 816) == 0
+
+
+def test_chain_create_rejects(L):
+    """Recorded chains validate exactly like emb_qlayer_seq, before touching the GPU."""
+    M = 1
+    good = (0, A, 128, 64, B, C)
+    h = ctypes.c_void_p(123)
+    arr = _layers([good])
+    assert L.emb_chain_create(arr, 1, M, None, 0, None) == emb.EMB_EINVAL
+    assert L.emb_chain_create(None, 1, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
+    assert h.value is None   # cleared on failure
+    assert L.emb_chain_create(arr, 0, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
+    chain = _layers([good, (0, A + (64 << 20), 128, 64, C, C + (1 << 20))])   # reads layer 0's Y
+    assert L.emb_chain_create(chain, 2, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
+    chain = _layers([good, (1, A + (64 << 20), 128, 64, B + 8, C + (1 << 20))])   # misaligned X
+    assert L.emb_chain_create(chain, 2, M, None, 0, ctypes.byref(h)) == emb.EMB_EALIGN
+    assert L.emb_chain_launch(None, None) == emb.EMB_EINVAL
+    assert L.emb_chain_destroy(None) == emb.EMB_OK
 
 
 def test_library_has_no_torch_dependency():

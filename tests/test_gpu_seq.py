@@ -100,3 +100,28 @@ def test_timeout_path_reports_status(cuda_device):
     assert emb.emb_device_status() == emb.EMB_OK   # cleared
     y = torch.ones(4, device="cuda") * 2
     assert y.sum().item() == 8.0
+
+
+@pytest.mark.parametrize("fmt,M", [(emb.EMB_Q8_0, 1), (emb.EMB_Q4_0, 1), (emb.EMB_Q8_0, 50),
+                                   (emb.EMB_Q4_0, 280)])
+def test_recorded_chain_replays(cuda_device, fmt, M):
+    """emb_chain_create records the chain's launches once; every replay reads the X
+    buffers as they are at launch time and gives the bits of emb_qlayer_seq."""
+    specs, _ = _decoder(fmt, M, 512, 128, 1536, 2, 3000 + M)
+    rec = emb.RecordedChain(specs, M)
+    xs = {sp[4].data_ptr(): sp[4] for sp in specs}
+    for it in range(3):
+        for j, x in enumerate(xs.values()):   # new activations in the same buffers
+            x.copy_(to_dev_bf16(activation_bits_np(M, x.shape[1], 50 * it + j)))
+        for sp in specs:
+            sp[5].fill_(float("nan"))
+        rec.launch()
+        torch.cuda.synchronize()
+        got = [sp[5].clone() for sp in specs]
+        emb.emb_qlayer_seq(specs, M)
+        torch.cuda.synchronize()
+        for i, sp in enumerate(specs):
+            assert torch.equal(got[i].view(torch.int32), sp[5].view(torch.int32)), (it, i)
+    assert emb.emb_device_status() == emb.EMB_OK
+    rec.close()
+    rec.close()   # idempotent
