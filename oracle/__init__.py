@@ -6,7 +6,7 @@ A plain, slow, obviously-correct restatement of the computation in C++
 import this package.  It shares no code with the CUDA library
 (``paper_2607_02501_gb300``) and neither imports the other.
 
-What it computes follows the paper's 8-bit / 4-bit weight configurations
+What it computes follows the paper's 8-, 6- and 4-bit weight configurations
 (Section 4 "Evaluation", Table 3); the block formats themselves are not given in
 the paper and are the readings stated in ``emb_oracle.cpp``'s header.
 """
@@ -25,6 +25,7 @@ _LIB_PATH = os.path.join(_OUT_DIR, "liboracle.so")
 
 Q8_0 = 0
 Q4_0 = 1
+Q6_0 = 2
 
 _lib = None
 
@@ -179,10 +180,32 @@ def qmatmul_sampled(fmt: int, img: np.ndarray, X_bf16_bits: np.ndarray, N: int, 
 
 
 def split_image(fmt: int, img: np.ndarray, N: int, K: int):
-    """Views of the codes plane and the scales plane (fp16 bits, [N][ldS]) of an image."""
-    codes_bytes = N * K if fmt == Q8_0 else N * K // 2
-    off = (codes_bytes + 255) // 256 * 256
+    """Views of the codes plane and the scales plane (fp16 bits, [N][ldS]) of an image.
+    For Q6_0 the codes "plane" is the low-nibble plane followed by the high-bits plane
+    (concatenated, without the padding between them)."""
     ldS = (K // 32 + 7) // 8 * 8
-    codes = img[:codes_bytes]
+    if fmt == Q6_0:
+        lo = N * K // 2
+        hoff = (lo + 255) // 256 * 256
+        off = (hoff + N * K // 4 + 255) // 256 * 256
+        codes = np.concatenate([img[:lo], img[hoff:hoff + N * K // 4]])
+    else:
+        codes_bytes = N * K if fmt == Q8_0 else N * K // 2
+        off = (codes_bytes + 255) // 256 * 256
+        codes = img[:codes_bytes]
     scales = img[off:off + N * ldS * 2].view(np.uint16).reshape(N, ldS)
     return codes, scales
+
+
+def q6_codes(img: np.ndarray, N: int, K: int) -> np.ndarray:
+    """The 6-bit codes [N][K] of a Q6_0 image, read back from its two planes."""
+    lo = N * K // 2
+    hoff = (lo + 255) // 256 * 256
+    L = img[:lo].reshape(N, K // 32, 16).astype(np.int64)
+    H = img[hoff:hoff + N * K // 4].reshape(N, K // 32, 8).astype(np.int64)
+    q = np.empty((N, K // 32, 32), dtype=np.int64)
+    q[:, :, :16] = L & 15
+    q[:, :, 16:] = L >> 4
+    for t in range(4):
+        q[:, :, 8 * t:8 * t + 8] |= ((H >> (2 * t)) & 3) << 4
+    return q.reshape(N, K)

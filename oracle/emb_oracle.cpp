@@ -6,20 +6,26 @@
 // no code, header, table or constant with the CUDA library and includes no CUDA
 // header; every conversion below is written out from the IEEE-754 definition.
 //
-// What is computed (the paper's 8-bit and 4-bit weight configurations, Section 4
-// "Evaluation", Table 3 columns "C++ 8-bit" / "C++ 4-bit"; the paper fixes no byte
-// format, so the block formats below are the readings listed in the design notes):
+// What is computed (the paper's 8-, 6- and 4-bit weight configurations, Section 4
+// "Evaluation", Table 3 columns "C++ 8-bit" / "C++ 6-bit" / "C++ 4-bit"; the paper fixes
+// no byte format, so the block formats below are the readings listed in the design notes):
 //   Q8_0: per 32 consecutive weights along K of one output row,
 //         d = fp16(max|w| / 127), q = clamp(round_half_away(w / d), -127, 127), w' = d*q
 //   Q4_0: m = the signed weight of largest magnitude (lowest index on ties),
 //         d = fp16(m / -8), q = clamp(round_half_away(w / d), -8, 7) + 8, w' = d*(q-8)
+//   Q6_0: the same with 6-bit codes: d = fp16(m / -32),
+//         q = clamp(round_half_away(w / d), -32, 31) + 32 in 0..63, w' = d*(q-32)
 //   matmul: Y[m][n] = sum_k w'[n][k] * x[m][k], accumulated in fp64, with the
 //         per-element tolerance bound B[m][n] = 1e-3 * sum_k |w'[n][k] x[m][k]| + 1e-6.
 //
 // Packed image (restated here from the layout definition, not shared with the GPU code):
 //   codes plane at byte 0: Q8_0 int8 [N][K]; Q4_0 uint8 [N][K/2] where, inside each
 //     32-block, byte j (0..15) holds code j in its low nibble and code j+16 in its high one;
-//   scales plane at byte roundup(codes_bytes, 256): fp16 [N][ldS], ldS = roundup(K/32, 8);
+//     Q6_0: the low 4 bits of each code in a plane laid out like Q4_0's ([N][K/2]), then at
+//     byte roundup(N*K/2, 256) the high 2 bits, uint8 [N][K/4], where inside each 32-block
+//     byte j (0..7) holds the high bits of codes j, j+8, j+16, j+24 at bits 0-1, 2-3, 4-5, 6-7;
+//   scales plane at byte roundup(codes_bytes, 256) (Q6_0: roundup of the end of the
+//     high-bits plane): fp16 [N][ldS], ldS = roundup(K/32, 8);
 //   every padding byte is zero.
 
 #include <cmath>
@@ -114,16 +120,18 @@ void ref_f32_to_bf16_n(const float* in, uint16_t* out, int64_t n) {
     for (int64_t i = 0; i < n; ++i) out[i] = ref_f32_to_bf16(in[i]);
 }
 
-// Byte size of the packed image (see header comment); 0 when the shape is invalid.
-int64_t ref_packed_bytes(int fmt, int64_t N, int64_t K) {
-    if ((fmt != 0 && fmt != 1) || N < 1 || K < 32 || K % 32) return 0;
-    int64_t codes = (fmt == 0) ? N * K : N * K / 2;
-    int64_t ldS = roundup(K / 32, 8);
-    return roundup(codes, 256) + N * ldS * 2;
-}
+// Q6_0: byte offset of the high-bits plane.
+static int64_t q6_high_offset(int64_t N, int64_t K) { return roundup(N * K / 2, 256); }
 
 static int64_t scales_offset(int fmt, int64_t N, int64_t K) {
+    if (fmt == 2) return roundup(q6_high_offset(N, K) + N * K / 4, 256);
     return roundup((fmt == 0) ? N * K : N * K / 2, 256);
+}
+
+// Byte size of the packed image (see header comment); 0 when the shape is invalid.
+int64_t ref_packed_bytes(int fmt, int64_t N, int64_t K) {
+    if ((fmt != 0 && fmt != 1 && fmt != 2) || N < 1 || K < 32 || K % 32) return 0;
+    return scales_offset(fmt, N, K) + N * roundup(K / 32, 8) * 2;
 }
 
 // Quantise fp32 W [N][K] into a zero-initialised packed image. Returns 0, or -1 if invalid.
@@ -152,19 +160,27 @@ int ref_quantize(int fmt, const float* W, int64_t N, int64_t K, uint8_t* out) {
                 int8_t* codes = reinterpret_cast<int8_t*>(out) + n * K + b * 32;
                 for (int i = 0; i < 32; ++i) codes[i] = int8_t(q[i]);
             } else {
+                // Q4_0 (half = 8) and Q6_0 (half = 32): codes q - half in [-half, half - 1]
+                const float half = (fmt == 1) ? 8.0f : 32.0f;
                 float amax = 0.0f, m = 0.0f;
                 for (int i = 0; i < 32; ++i)
                     if (std::fabs(w[i]) > amax) { amax = std::fabs(w[i]); m = w[i]; }
-                float d32 = m / -8.0f;
+                float d32 = m / -half;
                 dh = ref_f32_to_f16(d32);
                 float d = ref_f16_to_f32(dh);
                 for (int i = 0; i < 32; ++i) {
-                    if (d == 0.0f) { q[i] = 8; continue; }
+                    if (d == 0.0f) { q[i] = int(half); continue; }
                     float t = std::round(w[i] / d);
-                    q[i] = int(t < -8.0f ? -8.0f : (t > 7.0f ? 7.0f : t)) + 8;
+                    q[i] = int(t < -half ? -half : (t > half - 1.0f ? half - 1.0f : t)) + int(half);
                 }
                 uint8_t* codes = out + n * (K / 2) + b * 16;
-                for (int j = 0; j < 16; ++j) codes[j] = uint8_t(q[j] | (q[j + 16] << 4));
+                for (int j = 0; j < 16; ++j) codes[j] = uint8_t((q[j] & 15) | ((q[j + 16] & 15) << 4));
+                if (fmt == 2) {
+                    uint8_t* high = out + q6_high_offset(N, K) + n * (K / 4) + b * 8;
+                    for (int j = 0; j < 8; ++j)
+                        high[j] = uint8_t((q[j] >> 4) | ((q[j + 8] >> 4) << 2) | ((q[j + 16] >> 4) << 4) |
+                                          ((q[j + 24] >> 4) << 6));
+                }
             }
             scales[n * ldS + b] = dh;
         }
@@ -183,13 +199,17 @@ static void load_code(int fmt, const uint8_t* img, int64_t N, int64_t K, int64_t
         int64_t b = k / 32, i = k % 32;
         uint8_t byte = img[n * (K / 2) + b * 16 + (i % 16)];
         *q = (i < 16) ? (byte & 0xF) : (byte >> 4);
+        if (fmt == 2) {  // high 2 bits: byte i % 8 of the block, bit pair i / 8
+            uint8_t hb = img[q6_high_offset(N, K) + n * (K / 4) + b * 8 + (i % 8)];
+            *q |= ((hb >> (2 * (i / 8))) & 3) << 4;
+        }
     }
 }
 
-// w' as binary32: d*q (Q8_0) or d*(q-8) (Q4_0). The product of an 11-bit and an at most
-// 8-bit significand is exact in binary32.
+// w' as binary32: d*q (Q8_0), d*(q-8) (Q4_0) or d*(q-32) (Q6_0). The product of an 11-bit
+// and an at most 8-bit significand is exact in binary32.
 static float deq_value(int fmt, int q, float d) {
-    return fmt == 0 ? d * float(q) : d * float(q - 8);
+    return fmt == 0 ? d * float(q) : fmt == 1 ? d * float(q - 8) : d * float(q - 32);
 }
 
 int ref_dequant_f32(int fmt, const uint8_t* img, int64_t N, int64_t K, float* out) {

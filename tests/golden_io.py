@@ -39,8 +39,8 @@ def read_blocks(fname: str, default_code: int):
                 vals = [int(t) for t in val.split()]
                 c[:len(vals)] = vals
                 cur["codes"] = c
-            elif key == "bytes":
-                cur["bytes"] = np.array([int(t, 16) for t in val.split()], dtype=np.uint8)
+            elif key in ("bytes", "low", "high"):
+                cur[key] = np.array([int(t, 16) for t in val.split()], dtype=np.uint8)
             else:
                 raise ValueError(f"unknown key {key!r} in {fname}")
     return blocks

@@ -8,7 +8,7 @@ import pytest
 import torch
 
 import oracle
-from oracle import Q4_0, Q8_0
+from oracle import Q4_0, Q6_0, Q8_0
 from tests.golden_io import read_blocks
 from workloads import activation_bits_np, bf16_bits_np, weight_np
 
@@ -76,12 +76,17 @@ def test_bf16_rounding_matches_torch():
     (Q8_0, 1, 32, 256 + 16),
     # Q8_0 5x1152: 36 blocks -> pitch 40 halves; codes 5760 -> 5888
     (Q8_0, 5, 1152, 5888 + 5 * 40 * 2),
+    # Q6_0 3x96: low plane 144 B -> high plane at 256 (72 B, ends at 328) -> scales at 512
+    (Q6_0, 3, 96, 512 + 3 * 8 * 2),
+    # Q6_0 2048x2048: low 2097152 B, high 1048576 B (both 256-aligned), scales 2048 * 64 * 2
+    (Q6_0, 2048, 2048, 2097152 + 1048576 + 2048 * 64 * 2),
 ])
 def test_packed_bytes(fmt, N, K, expect):
     assert oracle.packed_bytes(fmt, N, K) == expect
 
 
-@pytest.mark.parametrize("fmt,N,K", [(2, 4, 32), (Q8_0, 0, 32), (Q8_0, 4, 48), (Q4_0, 4, 0)])
+@pytest.mark.parametrize("fmt,N,K", [(3, 4, 32), (-1, 4, 32), (Q8_0, 0, 32), (Q8_0, 4, 48),
+                                     (Q4_0, 4, 0), (Q6_0, 4, 48), (Q6_0, 0, 64)])
 def test_packed_bytes_rejects(fmt, N, K):
     assert oracle.packed_bytes(fmt, N, K) == 0
 
@@ -114,14 +119,33 @@ def test_q4_0_golden(blk):
     assert np.array_equal((c[:16] | (c[16:] << 4)).astype(np.uint8), blk["bytes"])
 
 
+@pytest.mark.parametrize("blk", read_blocks("q6_0_blocks.txt", 32), ids=lambda b: b["name"])
+def test_q6_0_golden(blk):
+    img = oracle.quantize(Q6_0, blk["w"].reshape(1, 32))
+    _, scales = oracle.split_image(Q6_0, img, 1, 32)
+    assert scales[0, 0] == blk["scale"], hex(scales[0, 0])
+    assert np.array_equal(img[:16], blk["low"]), img[:16]
+    assert np.array_equal(img[256:264], blk["high"]), img[256:264]
+    assert np.array_equal(oracle.q6_codes(img, 1, 32)[0], blk["codes"])
+    # padding (between the planes, before the scales, rest of the scale row) is zero
+    assert not img[16:256].any() and not img[264:512].any() and not scales[0, 1:].any()
+    # the listed codes agree with the listed bytes (fixture self-consistency)
+    c = blk["codes"]
+    assert np.array_equal(((c[:16] & 15) | ((c[16:] & 15) << 4)).astype(np.uint8), blk["low"])
+    h = (c[0:8] >> 4) | ((c[8:16] >> 4) << 2) | ((c[16:24] >> 4) << 4) | ((c[24:32] >> 4) << 6)
+    assert np.array_equal(h.astype(np.uint8), blk["high"])
+
+
 def test_golden_dequant_values():
-    """Dequantised values of the hand-worked blocks: d*q and d*(q-8) in exact arithmetic."""
-    for fmt, fname, dflt in ((Q8_0, "q8_0_blocks.txt", 0), (Q4_0, "q4_0_blocks.txt", 8)):
+    """Dequantised values of the hand-worked blocks: d*q, d*(q-8), d*(q-32) in exact
+    arithmetic."""
+    for fmt, fname, dflt in ((Q8_0, "q8_0_blocks.txt", 0), (Q4_0, "q4_0_blocks.txt", 8),
+                             (Q6_0, "q6_0_blocks.txt", 32)):
         for blk in read_blocks(fname, dflt):
             img = oracle.quantize(fmt, blk["w"].reshape(1, 32))
             deq = oracle.dequant_f32(fmt, img, 1, 32)[0].astype(np.float64)
             d = float(np.array([blk["scale"]], dtype=np.uint16).view(np.float16)[0])
-            q = blk["codes"].astype(np.float64) - (8 if fmt == Q4_0 else 0)
+            q = blk["codes"].astype(np.float64) - {Q8_0: 0, Q4_0: 8, Q6_0: 32}[fmt]
             assert np.array_equal(deq, d * q), blk["name"]
 
 
@@ -129,19 +153,21 @@ def test_golden_dequant_values():
 
 def _grid_weights(fmt, N, K, rng):
     """Weights that each format represents exactly: per block k_i * 2^e with a scale
-    that the quantiser recovers exactly (Q8_0: one |k|=127; Q4_0: first max is -8)."""
+    that the quantiser recovers exactly (Q8_0: one |k|=127; Q4_0 / Q6_0: the first
+    maximum is -8 / -32)."""
     e = rng.integers(-12, 3, size=(N, K // 32))
     if fmt == Q8_0:
         k = rng.integers(-127, 128, size=(N, K))
         k[:, ::32] = np.where(rng.random((N, K // 32)) < 0.5, 127, -127)
     else:
-        k = rng.integers(-7, 8, size=(N, K))
-        k[:, ::32] = -8
+        half = 8 if fmt == Q4_0 else 32
+        k = rng.integers(-half + 1, half, size=(N, K))
+        k[:, ::32] = -half
     w = k * np.exp2(np.repeat(e, 32, axis=1))
     return w.astype(np.float32), k
 
 
-@pytest.mark.parametrize("fmt", [Q8_0, Q4_0])
+@pytest.mark.parametrize("fmt", [Q8_0, Q4_0, Q6_0])
 def test_exact_grid_roundtrip(fmt):
     rng = np.random.default_rng(11)
     W, _ = _grid_weights(fmt, 9, 256, rng)
@@ -165,7 +191,7 @@ def _random_blocks(nblocks, rng, lo=1e-2, hi=1e3):
     return w.astype(np.float32)
 
 
-@pytest.mark.parametrize("fmt", [Q8_0, Q4_0])
+@pytest.mark.parametrize("fmt", [Q8_0, Q4_0, Q6_0])
 def test_roundtrip_invariant(fmt):
     rng = np.random.default_rng(3 + fmt)
     nb = 200_000
@@ -185,22 +211,25 @@ def test_roundtrip_invariant(fmt):
         assert (err[normal] <= d[normal] / 2 + slack[normal]).all()
     else:
         t = w / np.where(d == 0, 1, d)
-        # sign of d is -sign(m): codes are w/d with d signed; in-range means w/d in [-8.5, 7.5]
+        # sign of d is -sign(m): codes are w/d with d signed; in range means
+        # w/d in [-half - 0.5, half - 0.5] (half = 8 for Q4_0, 32 for Q6_0)
+        half = 8 if fmt == Q4_0 else 32
         dsigned = np.repeat(scales[:, :K // 32].view(np.float16).astype(np.float64), 32, axis=1)
         t = w / dsigned
-        inrange = normal & (t >= -8.5) & (t <= 7.5)
+        inrange = normal & (t >= -half - 0.5) & (t <= half - 0.5)
         assert inrange.mean() > 0.9
         assert (err[inrange] <= d[inrange] / 2 + slack[inrange]).all()
-        # out of range only on the side opposite to m, and by less than |d|(1 + 2^-8)
-        assert (t[normal] <= 8 * (1 + 2.0 ** -10)).all() and (t[normal] >= -8.5).all()
-        assert (err[normal] <= d[normal] * (1 + 2.0 ** -8) + slack[normal]).all()
+        # out of range only on the side opposite to m (|d| >= |m|/half (1 - 2^-11)), by less
+        # than |d| (1 + half 2^-11)
+        assert (t[normal] <= half * (1 + 2.0 ** -10)).all() and (t[normal] >= -half - 0.5).all()
+        assert (err[normal] <= d[normal] * (1 + half * 2.0 ** -11) + slack[normal]).all()
 
 
-@pytest.mark.parametrize("fmt", [Q8_0, Q4_0])
+@pytest.mark.parametrize("fmt", [Q8_0, Q4_0, Q6_0])
 def test_roundtrip_subnormal_scales(fmt):
     """Tiny blocks whose scale is an fp16 subnormal (or rounds to 0): the scale carries an
-    absolute rounding error of at most 2^-25, so the bound gains 127*2^-25 (Q8_0) or
-    8*2^-25 (Q4_0) on top of the normal-scale bounds."""
+    absolute rounding error of at most 2^-25, so the bound gains 127*2^-25 (Q8_0),
+    8*2^-25 (Q4_0) or 32*2^-25 (Q6_0) on top of the normal-scale bounds."""
     rng = np.random.default_rng(13 + fmt)
     W = _random_blocks(50_000, rng, lo=1e-9, hi=1e-4).reshape(-1, 32 * 50)
     N, K = W.shape
@@ -216,12 +245,14 @@ def test_roundtrip_subnormal_scales(fmt):
     if fmt == Q8_0:
         assert (err <= np.maximum(d / 2, 127 * 2.0 ** -25) + slack).all()
     else:
-        assert (err <= d + 8 * 2.0 ** -25 + slack).all()
+        half = 8 if fmt == Q4_0 else 32
+        assert (err <= d * (1 + half * 2.0 ** -11) + half * 2.0 ** -25 + slack).all()
 
 
-@pytest.mark.parametrize("fmt", [Q8_0, Q4_0])
+@pytest.mark.parametrize("fmt", [Q8_0, Q4_0, Q6_0])
 def test_scale_is_rounded_block_extreme(fmt):
-    """d is the fp16 rounding of max|w|/127 (Q8_0) or m/-8 (Q4_0), computed independently."""
+    """d is the fp16 rounding of max|w|/127 (Q8_0) or m/-8 (Q4_0) or m/-32 (Q6_0),
+    computed independently."""
     rng = np.random.default_rng(5)
     W = _random_blocks(20_000, rng).reshape(-1, 32 * 40)
     N, K = W.shape
@@ -233,7 +264,7 @@ def test_scale_is_rounded_block_extreme(fmt):
     else:
         idx = np.abs(blocks).argmax(axis=2)                  # first index of the maximum
         m = np.take_along_axis(blocks, idx[..., None], axis=2)[..., 0]
-        d32 = m / np.float32(-8)
+        d32 = m / np.float32(-8 if fmt == Q4_0 else -32)
     with np.errstate(over="ignore"):
         expect = d32.astype(np.float32).astype(np.float16).view(np.uint16)
     assert np.array_equal(scales[:, :K // 32], expect)
@@ -244,7 +275,7 @@ def test_codes_round_half_away_vs_numpy():
     rng = np.random.default_rng(9)
     W = _random_blocks(10_000, rng).reshape(-1, 32 * 25)
     N, K = W.shape
-    for fmt in (Q8_0, Q4_0):
+    for fmt in (Q8_0, Q4_0, Q6_0):
         img = oracle.quantize(fmt, W)
         codes, scales = oracle.split_image(fmt, img, N, K)
         d = np.repeat(scales[:, :K // 32].view(np.float16).astype(np.float32), 32, axis=1)
@@ -254,10 +285,13 @@ def test_codes_round_half_away_vs_numpy():
         if fmt == Q8_0:
             expect = np.where(d == 0, 0, np.clip(r, -127, 127)).astype(np.int64)
             got = codes.view(np.int8).reshape(N, K).astype(np.int64)
-        else:
+        elif fmt == Q4_0:
             expect = np.where(d == 0, 8, np.clip(r, -8, 7) + 8).astype(np.int64)
             b = codes.reshape(N, K // 32, 16)
             got = np.concatenate([b & 0xF, b >> 4], axis=2).reshape(N, K).astype(np.int64)
+        else:
+            expect = np.where(d == 0, 32, np.clip(r, -32, 31) + 32).astype(np.int64)
+            got = oracle.q6_codes(img, N, K)
         assert np.array_equal(got, expect)
 
 
@@ -282,7 +316,7 @@ def _exact_Y(W, Xf):
     return Y, A
 
 
-@pytest.mark.parametrize("fmt", [Q8_0, Q4_0])
+@pytest.mark.parametrize("fmt", [Q8_0, Q4_0, Q6_0])
 @pytest.mark.parametrize("M,N,K", [(1, 1, 32), (3, 4, 64), (4, 3, 32), (2, 2, 96)])
 def test_matmul_brute_force_exact(fmt, M, N, K):
     rng = np.random.default_rng(100 + M * 10 + N + K)
@@ -328,7 +362,7 @@ def test_matmul_orientation_identity():
     W[3, 3] = -s
     X = activation_bits_np(M, K, 4)
     xs = (X.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
-    for fmt in (Q8_0, Q4_0):
+    for fmt in (Q8_0, Q4_0, Q6_0):
         img = oracle.quantize(fmt, W)
         diag = np.diag(oracle.dequant_f32(fmt, img, N, K)).astype(np.float64)
         Y, _ = oracle.qmatmul(fmt, img, X, N, K)
@@ -338,12 +372,12 @@ def test_matmul_orientation_identity():
             d = float(np.float16(s / np.float32(127)))
             assert np.all(np.abs(diag) == 127 * d)
         else:
-            assert np.all(np.abs(diag) == s)            # s/8 = 0.09375 is exact in fp16
+            assert np.all(np.abs(diag) == s)            # s/8, s/32 are exact in fp16
 
 
 def test_matmul_matches_numpy_fp64():
     """Random shapes: the oracle's sequential fp64 sum vs numpy's fp64 matmul (BLAS)."""
-    for fmt in (Q8_0, Q4_0):
+    for fmt in (Q8_0, Q4_0, Q6_0):
         M, N, K = 5, 70, 320
         W = weight_np(N, K, 30 + fmt)
         X = activation_bits_np(M, K, 31 + fmt)
@@ -361,7 +395,7 @@ def test_threaded_and_sampled_agree():
     N, K, M = 37, 96, 3
     W = weight_np(N, K, 41)
     X = activation_bits_np(M, K, 42)
-    for fmt in (Q8_0, Q4_0):
+    for fmt in (Q8_0, Q4_0, Q6_0):
         img = oracle.quantize(fmt, W)
         Y1, B1 = oracle.qmatmul(fmt, img, X, N, K, nthreads=1)
         Y4, B4 = oracle.qmatmul(fmt, img, X, N, K, nthreads=4)
@@ -377,13 +411,18 @@ def test_quantize_rows_are_independent():
     (what the sampled full-size parity checks rely on)."""
     N, K = 12, 160
     W = weight_np(N, K, 51)
-    for fmt in (Q8_0, Q4_0):
+    for fmt in (Q8_0, Q4_0, Q6_0):
         full = oracle.quantize(fmt, W)
         cf, sf = oracle.split_image(fmt, full, N, K)
         rows = [0, 5, 11]
         sub = oracle.quantize(fmt, W[rows])
         cs, ss = oracle.split_image(fmt, sub, len(rows), K)
-        rb = K if fmt == Q8_0 else K // 2
+        planes = [(0, K)] if fmt == Q8_0 else [(0, K // 2)] if fmt == Q4_0 else \
+            [(0, K // 2), (N * K // 2, K // 4)]       # (plane start in cf, bytes per row)
         for i, r in enumerate(rows):
-            assert np.array_equal(cs[i * rb:(i + 1) * rb], cf[r * rb:(r + 1) * rb])
+            so = 0
+            for start, rb in planes:
+                sub_start = start * len(rows) // N
+                assert np.array_equal(cs[sub_start + i * rb:sub_start + (i + 1) * rb],
+                                      cf[start + r * rb:start + (r + 1) * rb])
             assert np.array_equal(ss[i], sf[r])
