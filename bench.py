@@ -165,6 +165,9 @@ WORKLOADS = {
     "single_linear": lambda: [wl.single_linear()],
     "action_expert": lambda: [wl.action_expert_denoise()],
     "gemma2b_prefill": lambda: [wl.gemma2b_prefill(wl.Q8_0), wl.gemma2b_prefill(wl.Q4_0)],
+    # the 6-bit configuration (Table 3, "C++ 6-bit"), decode and prefill
+    "gemma2b_decode_q6": lambda: [wl.gemma2b_decode(wl.Q6_0)],
+    "gemma2b_prefill_q6": lambda: [wl.gemma2b_prefill(wl.Q6_0)],
     "vit": lambda: [wl.vit_tower(wl.Q8_0), wl.vit_tower(wl.Q4_0)],
     "llama7b_decode": lambda: [wl.llama7b(1)],
     "llama7b_prefill": lambda: [wl.llama7b(280)],
@@ -267,7 +270,7 @@ def time_oracle(work, fmt, M, budget_s: float, min_rounds: int = 1):
     while True:
         for lin, img, X in work:
             oracle.qmatmul(fmt, img, X, lin.N, lin.K)
-            nbytes += lin.N * lin.K // 32 * (34 if fmt == wl.Q8_0 else 18) + M * lin.K * 2 + M * lin.N * 4
+            nbytes += lin.N * lin.K // 32 * wl.BLOCK_BYTES[fmt] + M * lin.K * 2 + M * lin.N * 4
         rounds += 1
         el = time.perf_counter() - t0
         if rounds >= min_rounds and el >= budget_s:
@@ -319,7 +322,7 @@ def run_reference(args):
         for w, items in work:
             for lin, img, X in items[:per_fmt]:
                 oracle.qmatmul(w.fmt, img, X, lin.N, lin.K)
-                nbytes += (lin.N * lin.K // 32 * (34 if w.fmt == wl.Q8_0 else 18)
+                nbytes += (lin.N * lin.K // 32 * wl.BLOCK_BYTES[w.fmt]
                            + w.M * lin.K * 2 + w.M * lin.N * 4)
     el = time.perf_counter() - t0
     value = nbytes / el / 1e9

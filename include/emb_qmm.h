@@ -9,12 +9,12 @@
  *     ("Latency-first closed-loop control"); Section 3.2, design principle 2
  *     ("Latency-first fused execution": graph replay, buffer reuse, operator
  *     fusion, careful host-device data movement);
- *   - the 8-bit and 4-bit weight configurations: Section 4 ("VLA model
- *     evaluation"), Table 3 columns "C++ 8-bit" / "C++ 4-bit";
+ *   - the 8-, 6- and 4-bit weight configurations: Section 4 ("VLA model
+ *     evaluation"), Table 3 columns "C++ 8-bit" / "C++ 6-bit" / "C++ 4-bit";
  *   - a stable deployment boundary behind one backend abstraction: abstract;
  *     Section 3.2 (Figure 2 description).
- * The paper gives no byte format; the two block formats below are this
- * library's definition of the 8-bit and 4-bit configurations.
+ * The paper gives no byte format; the three block formats below are this
+ * library's definition of the 8-, 6- and 4-bit configurations.
  *
  * Conventions for every entry point
  *   - W is [N][K] (output features x input features, PyTorch Linear.weight
@@ -60,7 +60,10 @@ typedef enum {
      * q in [0, 15]; w' = d * (q - 8). With m the signed weight of largest
      * magnitude (lowest index on ties): d = fp16_rne(m / -8),
      * q = clamp(round_half_away(w / d), -8, 7) + 8. */
-    EMB_Q4_0 = 1
+    EMB_Q4_0 = 1,
+    /* As EMB_Q4_0 with 6-bit codes q in [0, 63]: w' = d * (q - 32),
+     * d = fp16_rne(m / -32), q = clamp(round_half_away(w / d), -32, 31) + 32. */
+    EMB_Q6_0 = 2
 } emb_qfmt;
 
 typedef enum {
@@ -83,8 +86,13 @@ typedef enum {
  *     Q8_0: int8  [N][K], row-major;
  *     Q4_0: uint8 [N][K/2]; in each 32-weight block, byte j (0..15) holds
  *           code j in its low nibble and code j+16 in its high nibble;
- *   scales plane at byte roundup(codes_bytes, 256):
- *     fp16 [N][ldS] with ldS = roundup(K/32, 8) (16-byte row pitch);
+ *     Q6_0: the low 4 bits of every code in a [N][K/2] plane laid out as Q4_0's,
+ *           then, at byte roundup(N*K/2, 256), the high 2 bits: uint8 [N][K/4]
+ *           where in each block byte j (0..7) holds the high bits of codes j,
+ *           j+8, j+16, j+24 at bits 0-1, 2-3, 4-5, 6-7;
+ *   scales plane at byte roundup(codes_bytes, 256) (Q6_0: roundup of the end
+ *     of the high plane, 256): fp16 [N][ldS] with ldS = roundup(K/32, 8)
+ *     (16-byte row pitch);
  *   every padding byte is zero, so two images of the same weights compare equal
  *   byte for byte.
  * Returns the byte size, or 0 when fmt is unknown, N < 1, K < 32 or K % 32 != 0. */
@@ -99,6 +107,11 @@ EMB_API emb_status emb_quantize_q8_0(const float* W, int64_t N, int64_t K, void*
 
 /* As emb_quantize_q8_0 for EMB_Q4_0 (m/-8 must not overflow fp16). */
 EMB_API emb_status emb_quantize_q4_0(const float* W, int64_t N, int64_t K, void* W_blocks,
+                             emb_stream_t stream);
+
+/* As emb_quantize_q8_0 for EMB_Q6_0, the 6-bit configuration (Table 3, "C++ 6-bit";
+ * the paper gives no format, EMB_Q6_0 above is this library's definition). */
+EMB_API emb_status emb_quantize_q6_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream);
 
 /* ---------------------------------------------------------------------- matmul

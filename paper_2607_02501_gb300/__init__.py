@@ -23,6 +23,7 @@ HEADER_PATH = os.path.join(_HERE, "..", "include", "emb_qmm.h")
 
 EMB_Q8_0 = 0
 EMB_Q4_0 = 1
+EMB_Q6_0 = 2
 
 EMB_OK = 0
 EMB_EINVAL = 1
@@ -69,7 +70,7 @@ def lib():
     i64, i32, vp, sz = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t
     L.emb_qweight_bytes.argtypes = [i32, i64, i64]
     L.emb_qweight_bytes.restype = sz
-    for name in ("emb_quantize_q8_0", "emb_quantize_q4_0"):
+    for name in ("emb_quantize_q8_0", "emb_quantize_q4_0", "emb_quantize_q6_0"):
         getattr(L, name).argtypes = [vp, i64, i64, vp, vp]
         getattr(L, name).restype = i32
     L.emb_qmatmul.argtypes = [i32, vp, vp, vp, i64, i64, i64, vp]
@@ -144,6 +145,11 @@ def emb_quantize_q8_0(W, N: int, K: int, W_blocks, stream=None) -> None:
 def emb_quantize_q4_0(W, N: int, K: int, W_blocks, stream=None) -> None:
     _check(lib().emb_quantize_q4_0(_ptr(W), N, K, _ptr(W_blocks), _stream(stream)),
            "emb_quantize_q4_0")
+
+
+def emb_quantize_q6_0(W, N: int, K: int, W_blocks, stream=None) -> None:
+    _check(lib().emb_quantize_q6_0(_ptr(W), N, K, _ptr(W_blocks), _stream(stream)),
+           "emb_quantize_q6_0")
 
 
 def emb_qmatmul(fmt: int, W_blocks, X, Y, M: int, N: int, K: int, stream=None) -> None:
@@ -259,7 +265,8 @@ def quantize(fmt: int, W, stream=None):
     """Pack fp32 device W [N][K]; returns the packed image as a uint8 device tensor."""
     N, K = W.shape
     out = empty_qweight(fmt, N, K, device=W.device)
-    (emb_quantize_q8_0 if fmt == EMB_Q8_0 else emb_quantize_q4_0)(W, N, K, out, stream)
+    {EMB_Q8_0: emb_quantize_q8_0, EMB_Q4_0: emb_quantize_q4_0,
+     EMB_Q6_0: emb_quantize_q6_0}[fmt](W, N, K, out, stream)
     return out
 
 

@@ -41,7 +41,7 @@ struct Range {
 };
 bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi; }
 
-bool valid_fmt(int fmt) { return fmt == EMB_Q8_0 || fmt == EMB_Q4_0; }
+bool valid_fmt(int fmt) { return fmt == EMB_Q8_0 || fmt == EMB_Q4_0 || fmt == EMB_Q6_0; }
 
 bool valid_shape(int64_t M, int64_t N, int64_t K) {
     return M >= 1 && N >= 1 && K >= kQBlock && K % kQBlock == 0 && M < (int64_t(1) << 31) &&
@@ -68,7 +68,8 @@ emb_status check_layer(int fmt, const void* W, const uint16_t* X, const float* Y
 MatRef mat_ref(int fmt, const void* W, float* Y, int64_t N, int64_t K) {
     const Layout L = layout_of(fmt, N, K);
     const uint8_t* base = static_cast<const uint8_t*>(W);
-    return MatRef{base, reinterpret_cast<const __half*>(base + L.scales_off), Y, N};
+    return MatRef{base, reinterpret_cast<const __half*>(base + L.scales_off), Y, N,
+                  fmt == EMB_Q6_0 ? base + L.high_off : nullptr};
 }
 
 cudaError_t launch_group(const GroupRef& g, bool pdl, cudaStream_t s) {
@@ -129,6 +130,11 @@ emb_status emb_quantize_q8_0(const float* W, int64_t N, int64_t K, void* W_block
 emb_status emb_quantize_q4_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream) {
     return quantize_common(EMB_Q4_0, W, N, K, W_blocks, stream);
+}
+
+emb_status emb_quantize_q6_0(const float* W, int64_t N, int64_t K, void* W_blocks,
+                             emb_stream_t stream) {
+    return quantize_common(EMB_Q6_0, W, N, K, W_blocks, stream);
 }
 
 emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_t* X, float* Y, int64_t M,

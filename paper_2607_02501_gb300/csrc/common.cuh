@@ -16,7 +16,8 @@ __host__ __device__ inline int64_t roundup(int64_t a, int64_t b) { return (a + b
 
 // Byte layout of one packed image (the format comment of emb_qweight_bytes).
 struct Layout {
-    int64_t codes_bytes;  // codes plane size
+    int64_t codes_bytes;  // codes plane size (Q6_0: the low-nibble plane)
+    int64_t high_off;     // Q6_0: byte offset of the 2-bit high plane (256-aligned); else 0
     int64_t scales_off;   // byte offset of the fp16 scales plane (256-aligned)
     int64_t ldS;          // scales row pitch in halves (multiple of 8)
     int64_t total;        // total image size in bytes
@@ -25,7 +26,8 @@ struct Layout {
 __host__ __device__ inline Layout layout_of(int fmt, int64_t N, int64_t K) {
     Layout L;
     L.codes_bytes = (fmt == EMB_Q8_0) ? N * K : N * K / 2;
-    L.scales_off = roundup(L.codes_bytes, 256);
+    L.high_off = (fmt == EMB_Q6_0) ? roundup(L.codes_bytes, 256) : 0;
+    L.scales_off = (fmt == EMB_Q6_0) ? roundup(L.high_off + N * K / 4, 256) : roundup(L.codes_bytes, 256);
     L.ldS = roundup(K / kQBlock, 8);
     L.total = L.scales_off + N * L.ldS * 2;
     return L;
@@ -54,10 +56,11 @@ cudaError_t launch_dequant_bf16(int fmt, const void* img, int64_t N, int64_t K, 
 constexpr int kMaxGroup = 4;
 
 struct MatRef {
-    const uint8_t* codes;
+    const uint8_t* codes;   // Q6_0: the low-nibble plane
     const __half* scales;
     float* Y;
     int64_t N;
+    const uint8_t* high;    // Q6_0: the 2-bit high plane; else nullptr
 };
 
 struct GroupRef {

@@ -65,6 +65,7 @@ struct GemmParams {
     CUtensorMap x_map;                     // X [M][K] bf16, box {64, T}, 128B swizzle
     CUtensorMap codes_map[kMaxGroup];      // codes [N][row bytes] u8, box {128, 128}, 128B swizzle
     CUtensorMap scales_map[kMaxGroup];     // scales [N][ldS] u16, box {8, 128}
+    CUtensorMap high_map[kMaxGroup];       // Q6_0 high bits [N][K/4] u8, box {64, 128}, no swizzle
     float* Y[kMaxGroup];
     int32_t N[kMaxGroup];
     int32_t tile0[kMaxGroup + 1];
@@ -84,8 +85,11 @@ template <int FMT>
 struct RawTraits {
     static constexpr int planes = (FMT == EMB_Q8_0) ? 2 : 1;  // 128-byte code chunks per raw stage
     static constexpr int bytes = planes * kPlane;
+    // Q6_0: the high bits of a raw stage, 64 bytes per row (256 codes x 2 bits)
+    static constexpr int hbytes = (FMT == EMB_Q6_0) ? kBN * 64 : 0;
     // w' = d*(f - bias) where f = 2^15 + byte is built by __byte_perm
-    static constexpr float bias = (FMT == EMB_Q8_0) ? 32768.0f + 128.0f : 32768.0f + 8.0f;
+    static constexpr float bias = (FMT == EMB_Q8_0) ? 32768.0f + 128.0f
+                                : (FMT == EMB_Q4_0) ? 32768.0f + 8.0f : 32768.0f + 32.0f;
 };
 
 __device__ __forceinline__ uint4 lds128(const uint8_t* p) {
@@ -156,7 +160,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint8_t* x_ring = base;                                     // S x P x T x 128 B
     uint8_t* r_ring = x_ring + S * P * T * 128;                 // 2 x RT::bytes
     uint8_t* s_ring = r_ring + kRawStages * RT::bytes;          // 2 x 2 KB
-    uint64_t* bars = reinterpret_cast<uint64_t*>(s_ring + kRawStages * kScaleTile);
+    uint8_t* h_ring = s_ring + kRawStages * kScaleTile;          // Q6_0: 2 x 8 KB of high bits
+    uint64_t* bars = reinterpret_cast<uint64_t*>(h_ring + kRawStages * RT::hbytes);
     uint64_t* raw_full = bars;
     uint64_t* raw_empty = bars + kRawStages;
     uint64_t* x_full = bars + 2 * kRawStages;
@@ -204,6 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         ptx::prefetch_tmap(&p.x_map);
         ptx::prefetch_tmap(&p.codes_map[g]);
         ptx::prefetch_tmap(&p.scales_map[g]);
+        if constexpr (FMT == EMB_Q6_0) ptx::prefetch_tmap(&p.high_map[g]);
     }
     if (warp == 1) {
         ptx::tmem_alloc(tmem_slot, p.tmem_cols);
@@ -223,11 +229,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             auto issue_raw = [&](int r) {
                 const int slot = r % kRawStages;
                 const int rg = rs0 + r;  // raw stage index within the whole row
-                ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + kScaleTile);
+                ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + RT::hbytes + kScaleTile);
 #pragma unroll
                 for (int pl = 0; pl < RT::planes; ++pl)
                     ptx::tma_load_2d(r_ring + slot * RT::bytes + pl * kPlane, &p.codes_map[g],
                                      &raw_full[slot], (rg * RT::planes + pl) * 128, n0, pol_w);
+                if constexpr (FMT == EMB_Q6_0)  // x = 64 bytes per raw stage: 16-byte aligned
+                    ptx::tma_load_2d(h_ring + slot * RT::hbytes, &p.high_map[g], &raw_full[slot],
+                                     rg * 64, n0, pol_w);
                 ptx::tma_load_2d(s_ring + slot * kScaleTile, &p.scales_map[g], &raw_full[slot],
                                  rg * (kKR / kQBlock), n0, pol_w);
             };
@@ -385,11 +394,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     const int b = 2 * j + h;
                     const uint4 v = lds128(rbase + ((b ^ sx) << 4));
                     const uint32_t m = 0x0F0F0F0Fu;
+                    // Q4_0: the nibbles are the codes. Q6_0: OR in the high bits so that every
+                    // byte holds a whole code: high word (w & 1) >> 2(w >> 1) has the high bits
+                    // of low word w's codes at bits 0-1 (codes 4w+i) and 4-5 (codes 16+4w+i).
+                    uint32_t c0 = v.x & m, c1 = v.y & m, c2 = v.z & m, c3 = v.w & m;
+                    uint32_t e0 = (v.x >> 4) & m, e1 = (v.y >> 4) & m, e2 = (v.z >> 4) & m, e3 = (v.w >> 4) & m;
+                    if constexpr (FMT == EMB_Q6_0) {
+                        const uint2 hv = *reinterpret_cast<const uint2*>(h_ring + rs * RT::hbytes + t * 64 + b * 8);
+                        const uint32_t hw[4] = {hv.x, hv.y, hv.x >> 2, hv.y >> 2};
+                        c0 |= (hw[0] & 0x03030303u) << 4; e0 |= hw[0] & 0x30303030u;
+                        c1 |= (hw[1] & 0x03030303u) << 4; e1 |= hw[1] & 0x30303030u;
+                        c2 |= (hw[2] & 0x03030303u) << 4; e2 |= hw[2] & 0x30303030u;
+                        c3 |= (hw[3] & 0x03030303u) << 4; e3 |= hw[3] & 0x30303030u;
+                    }
                     uint4 hh[4], ll[4];
-                    make_chunk<SPLIT>(v.x & m, v.y & m, d[j], nbd[j], hh[0], ll[0]);               // codes 0..7
-                    make_chunk<SPLIT>(v.z & m, v.w & m, d[j], nbd[j], hh[1], ll[1]);               // 8..15
-                    make_chunk<SPLIT>((v.x >> 4) & m, (v.y >> 4) & m, d[j], nbd[j], hh[2], ll[2]); // 16..23
-                    make_chunk<SPLIT>((v.z >> 4) & m, (v.w >> 4) & m, d[j], nbd[j], hh[3], ll[3]); // 24..31
+                    make_chunk<SPLIT>(c0, c1, d[j], nbd[j], hh[0], ll[0]);  // codes 0..7
+                    make_chunk<SPLIT>(c2, c3, d[j], nbd[j], hh[1], ll[1]);  // 8..15
+                    make_chunk<SPLIT>(e0, e1, d[j], nbd[j], hh[2], ll[2]);  // 16..23
+                    make_chunk<SPLIT>(e2, e3, d[j], nbd[j], hh[3], ll[3]);  // 24..31
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {  // output chunk 4h+q -> columns 4q .. 4q+3
                         va[4 * q + 0] = hh[q].x; va[4 * q + 1] = hh[q].y;
@@ -547,7 +569,8 @@ constexpr int kOneCtaPerSm = 120 * 1024;
 
 template <int FMT, bool SPLIT>
 int smem_bytes(int T, int S, int P) {
-    const int need = 1024 + S * P * T * 128 + kRawStages * (RawTraits<FMT>::bytes + kScaleTile) +
+    const int need = 1024 + S * P * T * 128 +
+                     kRawStages * (RawTraits<FMT>::bytes + RawTraits<FMT>::hbytes + kScaleTile) +
                      (2 * kRawStages + 3 * S + 1) * 8 + 16;
     return need > kOneCtaPerSm ? need : kOneCtaPerSm;
 }
@@ -652,9 +675,10 @@ int pick_splits(int64_t tiles, int T, int64_t K, int stages, bool split_operand)
 
 }  // namespace
 
+// Q6_0's high plane ([N][K/4] bytes) needs a 16-byte row pitch for its tensor map.
 bool gemm_tc_supported(const GroupRef& g) {
     return g.M >= 1 && g.M <= int64_t(65535) * 256 && g.K <= (int64_t(1) << 30) &&
-           encode_fn() != nullptr;
+           (g.fmt != EMB_Q6_0 || g.K % 64 == 0) && encode_fn() != nullptr;
 }
 
 cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s) {
@@ -666,8 +690,9 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     const int64_t t_tiles = (g.M + 255) / 256;
     int T = int(roundup((g.M + t_tiles - 1) / t_tiles, 16));
     const bool split = g.K < 1024;
-    int S = g.fmt == EMB_Q8_0 ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
-                              : (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T));
+    int S = g.fmt == EMB_Q8_0   ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
+            : g.fmt == EMB_Q4_0 ? (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T))
+                                : (split ? pick_stages<EMB_Q6_0, true>(T) : pick_stages<EMB_Q6_0, false>(T));
     int splits = pick_splits(int64_t(t_tiles) * tiles, T, g.K, S, split);
     int P = 1, grid_x = int(t_tiles);
     // Two token tiles per CTA halve the dequantisation per token (each A tile feeds the MMAs
@@ -682,8 +707,9 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
         const int64_t t2 = 2 * ((g.M + 447) / 448);  // even count of tiles of at most 224
         const int T2 = int(roundup((g.M + t2 - 1) / t2, 16));
         int gap0 = 0, per_gap = 0;
-        const int S2 = (g.fmt == EMB_Q8_0) ? pick_stages_pair<EMB_Q8_0>(T2, gap0, per_gap)
-                                           : pick_stages_pair<EMB_Q4_0>(T2, gap0, per_gap);
+        const int S2 = (g.fmt == EMB_Q8_0)   ? pick_stages_pair<EMB_Q8_0>(T2, gap0, per_gap)
+                       : (g.fmt == EMB_Q4_0) ? pick_stages_pair<EMB_Q4_0>(T2, gap0, per_gap)
+                                             : pick_stages_pair<EMB_Q6_0>(T2, gap0, per_gap);
         const int sms = sm_count();
         if (S2 >= 2 && T2 <= 224 && sms > 0) {
             const double nk = double((g.K + kKC - 1) / kKC);
@@ -718,6 +744,11 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
                        uint64_t(g.ldS), uint64_t(mr.N), uint64_t(g.ldS) * 2, 8, kBN,
                        CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B))
             return cudaErrorInvalidValue;
+        if (g.fmt == EMB_Q6_0 &&
+            !encode_2d(&p.high_map[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, mr.high, uint64_t(g.K) / 4,
+                       uint64_t(mr.N), uint64_t(g.K) / 4, 64, kBN, CU_TENSOR_MAP_SWIZZLE_NONE,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B))
+            return cudaErrorInvalidValue;
         p.Y[i] = mr.Y;
         p.N[i] = int32_t(mr.N);
         p.tile0[i] = tiles;
@@ -737,9 +768,13 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
         return split    ? launch_kernel<EMB_Q8_0, true, 1>(p, grid_x, tiles, pdl, s)
                : P == 2 ? launch_kernel<EMB_Q8_0, false, 2>(p, grid_x, tiles, pdl, s)
                         : launch_kernel<EMB_Q8_0, false, 1>(p, grid_x, tiles, pdl, s);
-    return split    ? launch_kernel<EMB_Q4_0, true, 1>(p, grid_x, tiles, pdl, s)
-           : P == 2 ? launch_kernel<EMB_Q4_0, false, 2>(p, grid_x, tiles, pdl, s)
-                    : launch_kernel<EMB_Q4_0, false, 1>(p, grid_x, tiles, pdl, s);
+    if (g.fmt == EMB_Q4_0)
+        return split    ? launch_kernel<EMB_Q4_0, true, 1>(p, grid_x, tiles, pdl, s)
+               : P == 2 ? launch_kernel<EMB_Q4_0, false, 2>(p, grid_x, tiles, pdl, s)
+                        : launch_kernel<EMB_Q4_0, false, 1>(p, grid_x, tiles, pdl, s);
+    return split    ? launch_kernel<EMB_Q6_0, true, 1>(p, grid_x, tiles, pdl, s)
+           : P == 2 ? launch_kernel<EMB_Q6_0, false, 2>(p, grid_x, tiles, pdl, s)
+                    : launch_kernel<EMB_Q6_0, false, 1>(p, grid_x, tiles, pdl, s);
 }
 
 }  // namespace emb

@@ -29,6 +29,7 @@ namespace {
 
 struct GemvParams {
     const uint8_t* codes[kMaxGroup];
+    const uint8_t* high[kMaxGroup];  // Q6_0: 2-bit high plane of each matrix
     const __half* scales[kMaxGroup];
     float* Y[kMaxGroup];
     int32_t N[kMaxGroup];
@@ -43,6 +44,11 @@ __device__ __forceinline__ uint4 ld_stream_u4(const void* p) {
     asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
+    return v;
+}
+__device__ __forceinline__ uint2 ld_stream_u2(const void* p) {
+    uint2 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
     return v;
 }
 
@@ -118,6 +124,46 @@ __device__ __forceinline__ float dot_q4_unit(const uint4 c, const float* x) {
     return acc.x + acc.y;
 }
 
+// 32 Q6_0 codes (one block: 16 bytes of low nibbles c, 8 bytes of high bits h) times 32
+// fp32 activations -> sum of (q-32)*x. Low word j holds the low nibbles of codes 4j..4j+3
+// (bits 0-3 of its bytes) and 16+4j..16+4j+3 (bits 4-7); high word j&1 shifted right by
+// 2*(j>>1) holds their high bits at bits 0-1 and 4-5 of the same bytes. So every byte of
+// a = (c & 0x0F..) | (h & 0x03..) << 4 and of b = (c >> 4 & 0x0F..) | (h & 0x30..) is a
+// whole 6-bit code; __byte_perm(., 0x4B000000, 0x7540 + i) is 2^23 + q exactly and
+// subtracting 2^23 + 32 leaves q - 32 exactly.
+__device__ __forceinline__ float dot_q6_unit(const uint4 c, const uint2 h, const float* x) {
+    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
+    const float2 off = make_float2(-8388640.0f, -8388640.0f);  // -(2^23 + 32)
+    float2 acc = make_float2(0.0f, 0.0f);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const uint32_t hh = ((j & 1) ? h.y : h.x) >> (2 * (j >> 1));
+        const uint32_t a = and_or(w[j], 0x0F0F0F0Fu, (hh & 0x03030303u) << 4);
+        const uint32_t b = and_or(w[j] >> 4, 0x0F0F0F0Fu, hh & 0x30303030u);
+        const float2 a01 = __fadd2_rn(make_float2(__uint_as_float(__byte_perm(a, 0x4B000000u, 0x7540u)),
+                                                  __uint_as_float(__byte_perm(a, 0x4B000000u, 0x7541u))), off);
+        const float2 a23 = __fadd2_rn(make_float2(__uint_as_float(__byte_perm(a, 0x4B000000u, 0x7542u)),
+                                                  __uint_as_float(__byte_perm(a, 0x4B000000u, 0x7543u))), off);
+        const float2 b01 = __fadd2_rn(make_float2(__uint_as_float(__byte_perm(b, 0x4B000000u, 0x7540u)),
+                                                  __uint_as_float(__byte_perm(b, 0x4B000000u, 0x7541u))), off);
+        const float2 b23 = __fadd2_rn(make_float2(__uint_as_float(__byte_perm(b, 0x4B000000u, 0x7542u)),
+                                                  __uint_as_float(__byte_perm(b, 0x4B000000u, 0x7543u))), off);
+        acc = __ffma2_rn(a01, make_float2(x[4 * j + 0], x[4 * j + 1]), acc);
+        acc = __ffma2_rn(a23, make_float2(x[4 * j + 2], x[4 * j + 3]), acc);
+        acc = __ffma2_rn(b01, make_float2(x[16 + 4 * j + 0], x[16 + 4 * j + 1]), acc);
+        acc = __ffma2_rn(b23, make_float2(x[16 + 4 * j + 2], x[16 + 4 * j + 3]), acc);
+    }
+    return acc.x + acc.y;
+}
+
+// One 16-byte unit of codes (Q6_0: plus its 8 bytes of high bits) times its activations.
+template <int FMT>
+__device__ __forceinline__ float dot_unit(const uint4 c, const uint2 h, const float* x) {
+    if constexpr (FMT == EMB_Q8_0) return dot_q8_unit(c, x);
+    else if constexpr (FMT == EMB_Q4_0) return dot_q4_unit(c, x);
+    else return dot_q6_unit(c, h, x);
+}
+
 template <int FMT, int R, int NT, int MT>
 __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvParams p) {
     constexpr int UW = (FMT == EMB_Q8_0) ? 16 : 32;  // weights per 16-byte unit
@@ -133,28 +179,33 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
     const int t = threadIdx.x;
     const int64_t row_bytes = (FMT == EMB_Q8_0) ? int64_t(p.K) : int64_t(p.K) / 2;
     const uint8_t* cbase = p.codes[g] + int64_t(row0) * row_bytes;
+    const uint8_t* hbase = (FMT == EMB_Q6_0) ? p.high[g] + int64_t(row0) * (p.K / 4) : nullptr;
     const __half* sbase = p.scales[g] + int64_t(row0) * p.ldS;
     const int U = p.U;
 
     griddep_launch_dependents();
 
     uint4 c[R];
+    uint2 h[R];  // Q6_0 high bits (unused otherwise)
     float d[R];
-    auto load_unit = [&](int u, uint4* cc, float* dd) {
+    auto load_unit = [&](int u, uint4* cc, uint2* hh, float* dd) {
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             if (row0 + r < N) {
                 cc[r] = ld_stream_u4(cbase + r * row_bytes + int64_t(u) * 16);
+                if constexpr (FMT == EMB_Q6_0) hh[r] = ld_stream_u2(hbase + int64_t(r) * (p.K / 4) + int64_t(u) * 8);
+                else hh[r] = make_uint2(0, 0);
                 dd[r] = __half2float(sbase[int64_t(r) * p.ldS + ((FMT == EMB_Q8_0) ? (u >> 1) : u)]);
             } else {
                 cc[r] = make_uint4(0, 0, 0, 0);
+                hh[r] = make_uint2(0, 0);
                 dd[r] = 0.0f;
             }
         }
     };
 
     int u = t;
-    if (u < U) load_unit(u, c, d);
+    if (u < U) load_unit(u, c, h, d);
     // weights do not depend on earlier launches; X and Y may
     griddep_wait();
 
@@ -166,9 +217,10 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
 
     for (; u < U; u += NT) {
         uint4 cn[R];
+        uint2 hn[R];
         float dn[R];
         const int un = u + NT;
-        if (un < U) load_unit(un, cn, dn);
+        if (un < U) load_unit(un, cn, hn, dn);
 #pragma unroll
         for (int j = 0; j < MT; ++j) {
             const int m = m0 + j;
@@ -185,13 +237,13 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
             }
 #pragma unroll
             for (int r = 0; r < R; ++r) {
-                const float part = (FMT == EMB_Q8_0) ? dot_q8_unit(c[r], x) : dot_q4_unit(c[r], x);
+                const float part = dot_unit<FMT>(c[r], h[r], x);
                 acc[r][j] = fmaf(d[r], part, acc[r][j]);
             }
         }
         if (un < U) {
 #pragma unroll
-            for (int r = 0; r < R; ++r) { c[r] = cn[r]; d[r] = dn[r]; }
+            for (int r = 0; r < R; ++r) { c[r] = cn[r]; h[r] = hn[r]; d[r] = dn[r]; }
         }
     }
 
@@ -281,6 +333,7 @@ constexpr int kStageHeader = 1152;         // mbarriers (0..15), cross-warp sums
 
 struct StagedParams {
     const uint8_t* codes[kMaxGroup];
+    const uint8_t* high[kMaxGroup];  // Q6_0: 2-bit high plane of each matrix
     const __half* scales[kMaxGroup];
     float* Y[kMaxGroup];
     int32_t N[kMaxGroup];
@@ -300,9 +353,11 @@ __global__ void __launch_bounds__(kStageThreads) gemv_staged_kernel(const __grid
     uint64_t* bar_x = reinterpret_cast<uint64_t*>(smem + 8);  // activations landed
     float* red = reinterpret_cast<float*>(smem + 128);         // [WK][TR][MT]
     const int row_bytes = (FMT == EMB_Q8_0) ? p.K : p.K / 2;
+    const int high_bytes = (FMT == EMB_Q6_0) ? p.K / 4 : 0;               // Q6_0 high bits per row
     uint8_t* x_s = smem + kStageHeader;                                    // [MT][K] bf16
     uint8_t* codes_s = x_s + MT * p.K * 2;                                 // [TR][row_bytes]
-    uint8_t* scales_b = codes_s + uint32_t(p.TR) * uint32_t(row_bytes);    // [TR][ldS] fp16
+    uint8_t* high_s = codes_s + uint32_t(p.TR) * uint32_t(row_bytes);     // [TR][K/4] (Q6_0)
+    uint8_t* scales_b = high_s + uint32_t(p.TR) * uint32_t(high_bytes);   // [TR][ldS] fp16
     const __half* scales_s = reinterpret_cast<const __half*>(scales_b);
 
     const int tile = blockIdx.x;
@@ -318,12 +373,15 @@ __global__ void __launch_bounds__(kStageThreads) gemv_staged_kernel(const __grid
 
     if (threadIdx.x == 0) {
         const uint32_t codes_bytes = uint32_t(rows) * uint32_t(row_bytes);
+        const uint32_t hi_bytes = uint32_t(rows) * uint32_t(high_bytes);  // a multiple of 16 (K % 64 == 0)
         const uint32_t scales_bytes = uint32_t(rows) * uint32_t(p.ldS) * 2u;
         ptx::mbar_init(bar_w, 1);
         ptx::mbar_init(bar_x, 1);
         ptx::fence_mbar_init();
-        ptx::mbar_arrive_expect_tx(bar_w, codes_bytes + scales_bytes);
+        ptx::mbar_arrive_expect_tx(bar_w, codes_bytes + hi_bytes + scales_bytes);
         ptx::bulk_load(codes_s, p.codes[g] + int64_t(row0) * row_bytes, codes_bytes, bar_w);
+        if constexpr (FMT == EMB_Q6_0)
+            ptx::bulk_load(high_s, p.high[g] + int64_t(row0) * high_bytes, hi_bytes, bar_w);
         ptx::bulk_load(scales_b, p.scales[g] + int64_t(row0) * p.ldS, scales_bytes, bar_w);
     }
     ptx::griddep_launch_dependents();
@@ -357,11 +415,16 @@ __global__ void __launch_bounds__(kStageThreads) gemv_staged_kernel(const __grid
 #pragma unroll 2
         for (int u = u_lo + lane; u < u_hi; u += 32) {
             uint4 c[RW];
+            uint2 hq[RW];
             float d[RW];
 #pragma unroll
             for (int i = 0; i < RW; ++i) {
                 const int r = min(r0 + i, rows - 1);  // rows past the tile's end are never stored
                 c[i] = *reinterpret_cast<const uint4*>(codes_s + r * row_bytes + u * 16);
+                if constexpr (FMT == EMB_Q6_0)
+                    hq[i] = *reinterpret_cast<const uint2*>(high_s + r * high_bytes + u * 8);
+                else
+                    hq[i] = make_uint2(0, 0);
                 d[i] = __half2float(scales_s[r * p.ldS + ((FMT == EMB_Q8_0) ? (u >> 1) : u)]);
             }
 #pragma unroll
@@ -379,7 +442,7 @@ __global__ void __launch_bounds__(kStageThreads) gemv_staged_kernel(const __grid
                 }
 #pragma unroll
                 for (int i = 0; i < RW; ++i) {
-                    const float sdot = (FMT == EMB_Q8_0) ? dot_q8_unit(c[i], x) : dot_q4_unit(c[i], x);
+                    const float sdot = dot_unit<FMT>(c[i], hq[i], x);
                     acc[i][t] = fmaf(d[i], sdot, acc[i][t]);
                 }
             }
@@ -485,20 +548,26 @@ constexpr int64_t kStageMaxRowBytesM1 = 6 * 1024;
 
 bool launch_staged(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
     const int64_t row_bytes = (g.fmt == EMB_Q8_0) ? g.K : g.K / 2;
+    // Q6_0 rows also carry K/4 bytes of high bits, copied as a second contiguous block
+    // (16-byte multiples need K % 64 == 0; other K take the register path)
+    const int64_t high_bytes = (g.fmt == EMB_Q6_0) ? g.K / 4 : 0;
+    if (g.fmt == EMB_Q6_0 && g.K % 64 != 0) return false;
+    const int64_t weight_row_bytes = row_bytes + high_bytes;
     const int U = int((g.fmt == EMB_Q8_0) ? g.K / 16 : g.K / 32);
     const int MT = (g.M == 1) ? 1 : (g.M == 2) ? 2 : 4;
     if (int64_t(MT) * g.K * 2 > kStageXBytes) return false;
     int64_t rows = 0;
     for (int i = 0; i < g.n_mats; ++i) rows += g.mats[i].N;
-    if (rows * row_bytes < kStageMinBytes) return false;
-    if (g.M == 1 && row_bytes > kStageMaxRowBytesM1) return false;
+    if (rows * weight_row_bytes < kStageMinBytes) return false;
+    if (g.M == 1 && weight_row_bytes > kStageMaxRowBytesM1) return false;
     int RW = 0, WK = 0;
     const int64_t tile_bytes = (g.M == 1) ? kStageBytes / 2 : kStageBytes;
-    if (!pick_stage_shape(g.fmt, rows, row_bytes, U, tile_bytes, RW, WK)) return false;
+    if (!pick_stage_shape(g.fmt, rows, weight_row_bytes, U, tile_bytes, RW, WK)) return false;
     StagedParams p = {};
     const int TR = RW * kStageWarps / WK;
     int tiles = 0;
     for (int i = 0; i < g.n_mats; ++i) {
+        p.high[i] = g.mats[i].high;
         p.codes[i] = g.mats[i].codes;
         p.scales[i] = g.mats[i].scales;
         p.Y[i] = g.mats[i].Y;
@@ -516,11 +585,15 @@ bool launch_staged(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     p.WK = WK;
     p.X = g.X;
     p.status = status;
-    const size_t smem = kStageHeader + size_t(MT) * g.K * 2 + size_t(TR) * size_t(row_bytes + g.ldS * 2);
+    const size_t smem = kStageHeader + size_t(MT) * g.K * 2 + size_t(TR) * size_t(weight_row_bytes + g.ldS * 2);
     if (g.fmt == EMB_Q8_0) {
         if (MT == 1) err = launch_staged_rw<EMB_Q8_0, 1>(p, RW, tiles, smem, pdl, s);
         else if (MT == 2) err = launch_staged_rw<EMB_Q8_0, 2>(p, RW, tiles, smem, pdl, s);
         else err = launch_staged_rw<EMB_Q8_0, 4>(p, RW, tiles, smem, pdl, s);
+    } else if (g.fmt == EMB_Q6_0) {
+        if (MT == 1) err = launch_staged_rw<EMB_Q6_0, 1>(p, RW, tiles, smem, pdl, s);
+        else if (MT == 2) err = launch_staged_rw<EMB_Q6_0, 2>(p, RW, tiles, smem, pdl, s);
+        else err = launch_staged_rw<EMB_Q6_0, 4>(p, RW, tiles, smem, pdl, s);
     } else {
         if (MT == 1) err = launch_staged_rw<EMB_Q4_0, 1>(p, RW, tiles, smem, pdl, s);
         else if (MT == 2) err = launch_staged_rw<EMB_Q4_0, 2>(p, RW, tiles, smem, pdl, s);
@@ -790,6 +863,7 @@ cudaError_t launch_gemv_regs(const GroupRef& g, bool pdl, cudaStream_t s) {
     int tiles = 0;
     for (int i = 0; i < g.n_mats; ++i) {
         p.codes[i] = g.mats[i].codes;
+        p.high[i] = g.mats[i].high;
         p.scales[i] = g.mats[i].scales;
         p.Y[i] = g.mats[i].Y;
         p.N[i] = int32_t(g.mats[i].N);
@@ -809,9 +883,13 @@ cudaError_t launch_gemv_regs(const GroupRef& g, bool pdl, cudaStream_t s) {
         return R == 4 ? dispatch_nt<EMB_Q8_0, 4>(p, tiles, M, NT, pdl, s)
              : R == 2 ? dispatch_nt<EMB_Q8_0, 2>(p, tiles, M, NT, pdl, s)
                       : dispatch_nt<EMB_Q8_0, 1>(p, tiles, M, NT, pdl, s);
-    return R == 4 ? dispatch_nt<EMB_Q4_0, 4>(p, tiles, M, NT, pdl, s)
-         : R == 2 ? dispatch_nt<EMB_Q4_0, 2>(p, tiles, M, NT, pdl, s)
-                  : dispatch_nt<EMB_Q4_0, 1>(p, tiles, M, NT, pdl, s);
+    if (g.fmt == EMB_Q4_0)
+        return R == 4 ? dispatch_nt<EMB_Q4_0, 4>(p, tiles, M, NT, pdl, s)
+             : R == 2 ? dispatch_nt<EMB_Q4_0, 2>(p, tiles, M, NT, pdl, s)
+                      : dispatch_nt<EMB_Q4_0, 1>(p, tiles, M, NT, pdl, s);
+    return R == 4 ? dispatch_nt<EMB_Q6_0, 4>(p, tiles, M, NT, pdl, s)
+         : R == 2 ? dispatch_nt<EMB_Q6_0, 2>(p, tiles, M, NT, pdl, s)
+                  : dispatch_nt<EMB_Q6_0, 1>(p, tiles, M, NT, pdl, s);
 }
 
 }  // namespace emb

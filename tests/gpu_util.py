@@ -54,18 +54,24 @@ def run_case(fmt: int, M: int, N: int, K: int, seed: int):
 
 
 def layout_rows(fmt: int, img: torch.Tensor, N: int, K: int, rows) -> np.ndarray:
-    """The packed image restricted to the given rows (codes rows + scale rows), laid out
-    as the image of that row subset (what the oracle produces for W[rows])."""
+    """The packed image restricted to the given rows (codes rows, Q6_0 high-bit rows,
+    scale rows), laid out as the image of that row subset (what the oracle produces for
+    W[rows])."""
     rows = torch.as_tensor(np.asarray(rows), device=img.device, dtype=torch.long)
+    n = rows.numel()
     rb = K if fmt == emb.EMB_Q8_0 else K // 2
+    hb = K // 4 if fmt == emb.EMB_Q6_0 else 0
+    r256 = lambda v: (v + 255) // 256 * 256
     codes = img[:N * rb].view(N, rb)[rows]
-    off = (N * rb + 255) // 256 * 256
+    hoff, sub_hoff = r256(N * rb), r256(n * rb)
+    off = r256(hoff + N * hb) if hb else r256(N * rb)
+    sub_off = r256(sub_hoff + n * hb) if hb else r256(n * rb)
     ldS = (K // 32 + 7) // 8 * 8
     scales = img[off:off + N * ldS * 2].view(N, ldS * 2)[rows]
-    n = rows.numel()
-    sub_off = (n * rb + 255) // 256 * 256
     out = torch.zeros(sub_off + n * ldS * 2, dtype=torch.uint8, device=img.device)
     out[:n * rb] = codes.reshape(-1)
+    if hb:
+        out[sub_hoff:sub_hoff + n * hb] = img[hoff:hoff + N * hb].view(N, hb)[rows].reshape(-1)
     out[sub_off:] = scales.reshape(-1)
     return out.cpu().numpy()
 

@@ -17,7 +17,7 @@ def L():
 
 def test_every_declared_symbol_is_exported(L):
     names = emb.declared_symbols()
-    assert len(names) == 15
+    assert len(names) == 16
     for n in names:
         assert hasattr(L, n), n
 
@@ -30,14 +30,14 @@ def test_no_undeclared_exports(L):
     assert exported == set(emb.declared_symbols())
 
 
-@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0])
+@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0, emb.EMB_Q6_0])
 @pytest.mark.parametrize("N,K", [(1, 32), (3, 96), (2048, 2048), (256, 2048), (2048, 16384),
                                  (5, 1152), (4096, 11008), (129, 4608), (7, 4160)])
 def test_qweight_bytes_matches_oracle(L, fmt, N, K):
     assert emb.emb_qweight_bytes(fmt, N, K) == oracle.packed_bytes(fmt, N, K)
 
 
-@pytest.mark.parametrize("fmt,N,K", [(2, 4, 32), (-1, 4, 32), (0, 0, 32), (0, 4, 0), (0, 4, 48),
+@pytest.mark.parametrize("fmt,N,K", [(3, 4, 32), (-1, 4, 32), (0, 0, 32), (0, 4, 0), (0, 4, 48), (2, 4, 48),
                                      (1, -5, 64), (0, 4, 31)])
 def test_qweight_bytes_invalid(L, fmt, N, K):
     assert emb.emb_qweight_bytes(fmt, N, K) == 0
@@ -59,7 +59,8 @@ C = A + (2 << 30)
     ((0, None, B, C, 1, 128, 64), emb.EMB_EINVAL),          # null W
     ((0, A, None, C, 1, 128, 64), emb.EMB_EINVAL),          # null X
     ((0, A, B, None, 1, 128, 64), emb.EMB_EINVAL),          # null Y
-    ((2, A, B, C, 1, 128, 64), emb.EMB_EINVAL),             # unknown format
+    ((3, A, B, C, 1, 128, 64), emb.EMB_EINVAL),             # unknown format
+    ((2, A, B, C, 1, 128, 48), emb.EMB_EINVAL),             # Q6_0, K % 32
     ((0, A, B, C, 0, 128, 64), emb.EMB_EINVAL),             # M < 1
     ((0, A, B, C, 1, 0, 64), emb.EMB_EINVAL),               # N < 1
     ((0, A, B, C, 1, 128, 48), emb.EMB_EINVAL),             # K % 32
@@ -81,6 +82,9 @@ def test_quantize_rejects(L):
     assert L.emb_quantize_q8_0(B + 4, 4, 32, A, None) == emb.EMB_EALIGN
     assert L.emb_quantize_q4_0(B, 4, 32, A + 128, None) == emb.EMB_EALIGN
     assert L.emb_quantize_q8_0(A, 4, 32, A + 256, None) == emb.EMB_EINVAL   # in/out overlap
+    assert L.emb_quantize_q6_0(None, 4, 32, A, None) == emb.EMB_EINVAL
+    assert L.emb_quantize_q6_0(B, 4, 32, A + 16, None) == emb.EMB_EALIGN
+    assert L.emb_quantize_q6_0(A, 4, 64, A + 512, None) == emb.EMB_EINVAL   # in/out overlap
 
 
 def test_dequantize_rejects(L):

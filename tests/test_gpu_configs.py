@@ -54,7 +54,7 @@ def test_single_linear():
     print("max err/sum|wx|:", _run_workload(wl.single_linear()))
 
 
-@pytest.mark.parametrize("fmt", [wl.Q8_0, wl.Q4_0])
+@pytest.mark.parametrize("fmt", [wl.Q8_0, wl.Q4_0, wl.Q6_0])
 def test_gemma2b_decode(fmt):
     print("max err/sum|wx|:", _run_workload(wl.gemma2b_decode(fmt)))
 
@@ -63,7 +63,7 @@ def test_action_expert_denoise():
     print("max err/sum|wx|:", _run_workload(wl.action_expert_denoise()))
 
 
-@pytest.mark.parametrize("fmt", [wl.Q8_0, wl.Q4_0])
+@pytest.mark.parametrize("fmt", [wl.Q8_0, wl.Q4_0, wl.Q6_0])
 def test_gemma2b_prefill(fmt):
     toks = np.unique(np.r_[0, 255, 256, 767, 768, 815, np.random.default_rng(1).choice(816, 10)])
     print("max err/sum|wx|:", _run_workload(wl.gemma2b_prefill(fmt), layers=4, token_sample=toks))

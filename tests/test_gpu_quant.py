@@ -32,7 +32,7 @@ def _adversarial(N, K, seed):
     return W
 
 
-@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0])
+@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0, emb.EMB_Q6_0])
 @pytest.mark.parametrize("N,K", SHAPES)
 def test_pack_bit_exact(cuda_device, fmt, N, K):
     W = _adversarial(N, K, 100 + N + K)
@@ -44,7 +44,8 @@ def test_pack_bit_exact(cuda_device, fmt, N, K):
 
 
 @pytest.mark.parametrize("fmt,fname,dflt", [(emb.EMB_Q8_0, "q8_0_blocks.txt", 0),
-                                            (emb.EMB_Q4_0, "q4_0_blocks.txt", 8)])
+                                            (emb.EMB_Q4_0, "q4_0_blocks.txt", 8),
+                                            (emb.EMB_Q6_0, "q6_0_blocks.txt", 32)])
 def test_pack_golden_blocks(cuda_device, fmt, fname, dflt):
     blocks = read_blocks(fname, dflt)
     W = np.stack([b["w"] for b in blocks]).astype(np.float32)   # one row per block
@@ -54,11 +55,15 @@ def test_pack_golden_blocks(cuda_device, fmt, fname, dflt):
         assert scales[i, 0] == b["scale"], b["name"]
         if fmt == emb.EMB_Q8_0:
             assert np.array_equal(codes[32 * i:32 * i + 32].view(np.int8), b["codes"]), b["name"]
-        else:
+        elif fmt == emb.EMB_Q4_0:
             assert np.array_equal(codes[16 * i:16 * i + 16], b["bytes"]), b["name"]
+        else:   # low plane (16 bytes per block), then the high plane (8 bytes per block)
+            n = len(blocks)
+            assert np.array_equal(codes[16 * i:16 * i + 16], b["low"]), b["name"]
+            assert np.array_equal(codes[16 * n + 8 * i:16 * n + 8 * i + 8], b["high"]), b["name"]
 
 
-@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0])
+@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0, emb.EMB_Q6_0])
 @pytest.mark.parametrize("N,K", [(3, 96), (136, 1152), (64, 4096)])
 def test_dequant_bit_exact(cuda_device, fmt, N, K):
     W = _adversarial(N, K, 7 + K)

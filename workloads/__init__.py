@@ -20,7 +20,9 @@ import numpy as np
 
 Q8_0 = 0
 Q4_0 = 1
-FMT_NAMES = {Q8_0: "Q8_0", Q4_0: "Q4_0"}
+Q6_0 = 2
+FMT_NAMES = {Q8_0: "Q8_0", Q4_0: "Q4_0", Q6_0: "Q6_0"}
+BLOCK_BYTES = {Q8_0: 34, Q4_0: 18, Q6_0: 26}   # packed bytes per 32 weights (codes + fp16 scale)
 
 
 @dataclasses.dataclass(frozen=True)
@@ -52,7 +54,7 @@ class Workload:
         return sum(l.N * l.K for l in self.linears())
 
     def weight_bytes(self) -> int:
-        per = 34 if self.fmt == Q8_0 else 18
+        per = BLOCK_BYTES[self.fmt]
         return sum(l.N * l.K // 32 * per for l in self.linears())
 
     def algorithmic_bytes(self) -> int:
