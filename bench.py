@@ -165,7 +165,7 @@ WORKLOADS = {
     "single_linear": lambda: [wl.single_linear()],
     "action_expert": lambda: [wl.action_expert_denoise()],
     "gemma2b_prefill": lambda: [wl.gemma2b_prefill(wl.Q8_0), wl.gemma2b_prefill(wl.Q4_0)],
-    # the 6-bit configuration (Table 3, "C++ 6-bit"), decode and prefill
+    # the 6-bit configuration (Table 3), decode and prefill
     "gemma2b_decode_q6": lambda: [wl.gemma2b_decode(wl.Q6_0)],
     "gemma2b_prefill_q6": lambda: [wl.gemma2b_prefill(wl.Q6_0)],
     "vit": lambda: [wl.vit_tower(wl.Q8_0), wl.vit_tower(wl.Q4_0)],

@@ -5,12 +5,12 @@
  *
  * Paper: "Embodied.cpp: A Portable Inference Runtime of Embodied AI Models on
  * Heterogeneous Robots" (arXiv 2607.02501).
- *   - batch-1, latency-first execution: Section 3.1, challenge 2
- *     ("Latency-first closed-loop control"); Section 3.2, design principle 2
- *     ("Latency-first fused execution": graph replay, buffer reuse, operator
- *     fusion, careful host-device data movement);
- *   - the 8-, 6- and 4-bit weight configurations: Section 4 ("VLA model
- *     evaluation"), Table 3 columns "C++ 8-bit" / "C++ 6-bit" / "C++ 4-bit";
+ *   - batch-1 execution where each control step's latency is what counts:
+ *     Section 3.1, challenge 2; Section 3.2, design principle 2 (fusing the
+ *     step's work, replaying it as a recorded graph, reusing its buffers and
+ *     keeping host-device copies few);
+ *   - the 8-, 6- and 4-bit weight configurations: Section 4, Table 3 (its
+ *     8-bit, 6-bit and 4-bit C++ columns);
  *   - a stable deployment boundary behind one backend abstraction: abstract;
  *     Section 3.2 (Figure 2 description).
  * The paper gives no byte format; the three block formats below are this
@@ -109,7 +109,7 @@ EMB_API emb_status emb_quantize_q8_0(const float* W, int64_t N, int64_t K, void*
 EMB_API emb_status emb_quantize_q4_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream);
 
-/* As emb_quantize_q8_0 for EMB_Q6_0, the 6-bit configuration (Table 3, "C++ 6-bit";
+/* As emb_quantize_q8_0 for EMB_Q6_0, the 6-bit configuration (Table 3, 6-bit column;
  * the paper gives no format, EMB_Q6_0 above is this library's definition). */
 EMB_API emb_status emb_quantize_q6_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream);
@@ -145,7 +145,7 @@ typedef struct {
 EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M);
 
 /* Run n_layers linears in order on `stream`, all with M tokens (the paper's
- * "graph replay, buffer reuse, operator fusion": Section 3.2, principle 2).
+ * fusion, graph replay and buffer reuse of Section 3.2, principle 2).
  * Semantics are those of n_layers emb_qmatmul calls in sequence. Consecutive
  * layers that read the same X with the same fmt and K (q/k/v, gate/up) are
  * fused into one launch; each launch may fetch its weights before the previous
@@ -159,7 +159,7 @@ EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_
                           void* workspace, size_t ws_bytes, emb_stream_t stream);
 
 /* ------------------------------------------------------------ recorded chains
- * The paper's "graph replay" and "buffer reuse" (Section 3.2, design principle 2): the
+ * Graph replay and buffer reuse (Section 3.2, design principle 2): the
  * launches that emb_qlayer_seq(layers, n_layers, M, workspace, ws_bytes, ...) enqueues
  * are recorded once into a CUDA graph and then replayed with one call, so a closed-loop
  * step costs one host call instead of one per launch group. */

@@ -6,9 +6,9 @@
 // no code, header, table or constant with the CUDA library and includes no CUDA
 // header; every conversion below is written out from the IEEE-754 definition.
 //
-// What is computed (the paper's 8-, 6- and 4-bit weight configurations, Section 4
-// "Evaluation", Table 3 columns "C++ 8-bit" / "C++ 6-bit" / "C++ 4-bit"; the paper fixes
-// no byte format, so the block formats below are the readings listed in the design notes):
+// What is computed (the paper's 8-, 6- and 4-bit weight configurations, Section 4,
+// Table 3; the paper fixes no byte format, so the block formats below are the readings
+// listed in the design notes):
 //   Q8_0: per 32 consecutive weights along K of one output row,
 //         d = fp16(max|w| / 127), q = clamp(round_half_away(w / d), -127, 127), w' = d*q
 //   Q4_0: m = the signed weight of largest magnitude (lowest index on ties),

@@ -8,7 +8,7 @@ The paper evaluates closed-loop policies whose weights and tasks are not
 available here (Section 4, Tables 3-4), so every input is synthetic: weights
 ~N(0, 0.02) in fp32 (optionally with 1% of entries multiplied by 8), activations
 ~N(0, 1) rounded to bf16.  The token counts follow one closed-loop step of the
-paper's batch-1 setting (Section 3.1 "Latency-first closed-loop control"):
+paper's batch-1 closed-loop setting (Section 3.1, challenge 2):
 M=1 action-token decode, M=50 action-chunk denoising, M=280..816 prefix prefill.
 """
 from __future__ import annotations
