@@ -209,3 +209,62 @@ def q6_codes(img: np.ndarray, N: int, K: int) -> np.ndarray:
     for t in range(4):
         q[:, :, 8 * t:8 * t + 8] |= ((H >> (2 * t)) & 3) << 4
     return q.reshape(N, K)
+
+
+# ---------------------------------------------------------------------- epilogues
+# Per-layer output transforms of a layer chain (this build's fused epilogues; the paper
+# describes fused execution in Section 3.2, principle 2, without fixing any). Plain fp64
+# definitions on top of the fp64 matmul reference Y and its bound B.
+
+EPI_F32, EPI_BF16, EPI_ADD, EPI_GEGLU, EPI_SWIGLU = 0, 1, 2, 3, 4
+
+
+def gelu_tanh(g):
+    """GELU in its tanh form: 0.5 g (1 + tanh(sqrt(2/pi) (g + 0.044715 g^3))), fp64."""
+    g = np.asarray(g, dtype=np.float64)
+    return 0.5 * g * (1.0 + np.tanh(np.sqrt(2.0 / np.pi) * (g + 0.044715 * g ** 3)))
+
+
+def silu(g):
+    """SiLU: g * sigmoid(g) = g / (1 + exp(-g)), fp64."""
+    g = np.asarray(g, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        return g / (1.0 + np.exp(-g))
+
+
+def bf16_round(y):
+    """fp64 values rounded to bfloat16 (via binary32, nearest even) and back, fp64."""
+    b = f32_to_bf16_bits(np.asarray(y, dtype=np.float32))
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def epilogue_reference(kind: int, Y, B, R=None):
+    """Reference output and per-element bound of one layer with epilogue `kind`.
+
+    Y, B: the fp64 matmul reference and its bound ([M][N]); R: the fp32 values already
+    in the output buffer (EPI_ADD only). Gated kinds take the rows of W interleaved as
+    (gate_0, up_0, gate_1, up_1, ...) and give [M][N/2]: act(gate) * up.
+    Bounds (the fp32 result acc satisfies |acc - Y| <= B):
+      EPI_F32:   B
+      EPI_BF16:  B + 2^-8 (|Y| + B)                     one bf16 rounding of acc
+      EPI_ADD:   B + 2^-23 (|R| + |Y| + B)              one fp32 rounding of R + acc
+      gated:     |act(g)| B_u + (|u| + B_u) (1.2 B_g + 2^-20 (|g| + B_g + 1))
+                 + 2^-8 |h| + 1e-6                      act' <= 1.2 for both activations;
+                 fp32 evaluation of act within 2^-20 (|g| + 1); one bf16 rounding of h
+    """
+    Y = np.asarray(Y, dtype=np.float64)
+    B = np.asarray(B, dtype=np.float64)
+    if kind == EPI_F32:
+        return Y, B
+    if kind == EPI_BF16:
+        return Y, B + 2.0 ** -8 * (np.abs(Y) + B)
+    if kind == EPI_ADD:
+        R = np.asarray(R, dtype=np.float64)
+        return R + Y, B + 2.0 ** -23 * (np.abs(R) + np.abs(Y) + B)
+    g, u = Y[:, 0::2], Y[:, 1::2]
+    Bg, Bu = B[:, 0::2], B[:, 1::2]
+    act = gelu_tanh(g) if kind == EPI_GEGLU else silu(g)
+    h = act * u
+    bound = (np.abs(act) * Bu + (np.abs(u) + Bu) * (1.2 * Bg + 2.0 ** -20 * (np.abs(g) + Bg + 1.0))
+             + 2.0 ** -8 * np.abs(h) + 1e-6)
+    return h, bound
