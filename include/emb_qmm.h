@@ -128,14 +128,32 @@ EMB_API emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_
 
 /* --------------------------------------------------------------- layer chains
  * One linear layer of a chain: Y = X x w'^T with its own X and Y (device). */
+/* What a layer of a chain writes (its epilogue). acc[m][n] is the fp32 result
+ * sum_k w'[n][k] x[m][k] with emb_qmatmul's accuracy.
+ *   EMB_EPI_F32    Y fp32 [M][N] = acc                       (emb_qmatmul's output)
+ *   EMB_EPI_BF16   Y bf16 [M][N] = bf16_rne(acc)             (input of a next layer)
+ *   EMB_EPI_ADD    Y fp32 [M][N] += acc, one fp32 rounding   (residual add in place)
+ *   EMB_EPI_GEGLU  W holds gate and up rows interleaved (row 2i = gate_i, row 2i+1 =
+ *                  up_i; N even); Y bf16 [M][N/2] = bf16_rne(gelu(acc[2i]) * acc[2i+1])
+ *                  with gelu(g) = 0.5 g (1 + tanh(sqrt(2/pi) (g + 0.044715 g^3)))
+ *   EMB_EPI_SWIGLU as EMB_EPI_GEGLU with silu(g) = g / (1 + exp(-g))
+ * The activations are evaluated in fp32 with the CUDA math library. */
+typedef enum {
+    EMB_EPI_F32 = 0,
+    EMB_EPI_BF16 = 1,
+    EMB_EPI_ADD = 2,
+    EMB_EPI_GEGLU = 3,
+    EMB_EPI_SWIGLU = 4
+} emb_epilogue;
+
 typedef struct {
     int32_t fmt;            /* emb_qfmt */
-    int32_t reserved;       /* must be 0 */
+    int32_t epilogue;       /* emb_epilogue */
     const void* W_blocks;   /* packed image of W [N][K] */
     int64_t N;
     int64_t K;
     const uint16_t* X;      /* [M][K] bf16 */
-    float* Y;               /* [M][N] fp32 */
+    void* Y;                /* as the epilogue says; 16-byte aligned */
 } emb_qlayer;
 
 #define EMB_MAX_LAYERS 4096
@@ -146,12 +164,16 @@ EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, 
 
 /* Run n_layers linears in order on `stream`, all with M tokens (the paper's
  * fusion, graph replay and buffer reuse of Section 3.2, principle 2).
- * Semantics are those of n_layers emb_qmatmul calls in sequence. Consecutive
- * layers that read the same X with the same fmt and K (q/k/v, gate/up) are
- * fused into one launch; each launch may fetch its weights before the previous
- * launch has finished (programmatic dependent launch), and reads X only after
- * it. A layer's X or W_blocks may not overlap the Y of the same or an earlier
- * layer inside one call (EMB_EINVAL). The call enqueues kernels only (plus
+ * Semantics are those of n_layers single-layer calls in sequence, each with
+ * its epilogue. Consecutive layers that read the same X with the same fmt, K
+ * and epilogue (q/k/v, gate/up) are fused into one launch; each launch may
+ * fetch its weights before the previous launch has finished (programmatic
+ * dependent launch), and reads X and writes Y only after it. So a layer's X may
+ * be the output of an earlier layer of the same call (a bf16 epilogue feeding
+ * the next projection), and layers may add into the same residual buffer in
+ * turn. A layer's W_blocks may not overlap the Y of the same or an earlier
+ * layer, and its X may not overlap its own Y (EMB_EINVAL); an unknown epilogue,
+ * or a gated one with odd N, is EMB_EINVAL. The call enqueues kernels only (plus
  * memsets of the workspace), so it may be captured into a CUDA graph and
  * replayed. workspace: device, 256-byte aligned, >= emb_qlayer_seq_workspace()
  * bytes (may be NULL when that is 0). */

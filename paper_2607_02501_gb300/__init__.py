@@ -34,6 +34,13 @@ EMB_ETIMEOUT = 5
 EMB_EUNSUPPORTED = 6
 EMB_MAX_LAYERS = 4096
 
+# layer epilogues (emb_epilogue)
+EMB_EPI_F32 = 0
+EMB_EPI_BF16 = 1
+EMB_EPI_ADD = 2
+EMB_EPI_GEGLU = 3
+EMB_EPI_SWIGLU = 4
+
 _STATUS_NAMES = {0: "EMB_OK", 1: "EMB_EINVAL", 2: "EMB_EALIGN", 3: "EMB_ENOSPC",
                  4: "EMB_ECUDA", 5: "EMB_ETIMEOUT", 6: "EMB_EUNSUPPORTED"}
 
@@ -45,7 +52,7 @@ class EmbError(RuntimeError):
 
 
 class emb_qlayer(ctypes.Structure):
-    _fields_ = [("fmt", ctypes.c_int32), ("reserved", ctypes.c_int32),
+    _fields_ = [("fmt", ctypes.c_int32), ("epilogue", ctypes.c_int32),
                 ("W_blocks", ctypes.c_void_p), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
                 ("X", ctypes.c_void_p), ("Y", ctypes.c_void_p)]
 
@@ -158,10 +165,12 @@ def emb_qmatmul(fmt: int, W_blocks, X, Y, M: int, N: int, K: int, stream=None) -
 
 
 def make_layers(specs: Sequence) -> ctypes.Array:
-    """specs: iterable of (fmt, W_blocks, N, K, X, Y) -> a C array of emb_qlayer."""
+    """specs: iterable of (fmt, W_blocks, N, K, X, Y[, epilogue]) -> a C array of emb_qlayer."""
     arr = (emb_qlayer * len(specs))()
-    for i, (fmt, W, N, K, X, Y) in enumerate(specs):
-        arr[i] = emb_qlayer(fmt, 0, _ptr(W), N, K, _ptr(X), _ptr(Y))
+    for i, sp in enumerate(specs):
+        fmt, W, N, K, X, Y = sp[:6]
+        epi = sp[6] if len(sp) > 6 else EMB_EPI_F32
+        arr[i] = emb_qlayer(fmt, epi, _ptr(W), N, K, _ptr(X), _ptr(Y))
     return arr
 
 

@@ -51,21 +51,31 @@ bool valid_shape(int64_t M, int64_t N, int64_t K) {
 
 emb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? EMB_OK : EMB_ECUDA; }
 
+bool valid_epi(int epi) { return epi >= EMB_EPI_F32 && epi <= EMB_EPI_SWIGLU; }
+
+// Bytes a layer's epilogue writes (and, for EMB_EPI_ADD, reads) at Y.
+int64_t y_bytes(int epi, int64_t M, int64_t N) {
+    if (epi == EMB_EPI_F32 || epi == EMB_EPI_ADD) return M * N * 4;
+    if (epi == EMB_EPI_BF16) return M * N * 2;
+    return M * (N / 2) * 2;  // gated: one bf16 per gate/up row pair
+}
+
 // Validation shared by emb_qmatmul and every layer of emb_qlayer_seq.
-emb_status check_layer(int fmt, const void* W, const uint16_t* X, const float* Y, int64_t M,
+emb_status check_layer(int fmt, int epi, const void* W, const uint16_t* X, const void* Y, int64_t M,
                        int64_t N, int64_t K) {
-    if (!valid_fmt(fmt) || !valid_shape(M, N, K)) return EMB_EINVAL;
+    if (!valid_fmt(fmt) || !valid_epi(epi) || !valid_shape(M, N, K)) return EMB_EINVAL;
+    if (epi >= EMB_EPI_GEGLU && N % 2 != 0) return EMB_EINVAL;
     if (!W || !X || !Y) return EMB_EINVAL;
     if (!aligned(W, 256) || !aligned(X, 16) || !aligned(Y, 16)) return EMB_EALIGN;
     const Layout L = layout_of(fmt, N, K);
     const Range rw{uintptr_t(W), uintptr_t(W) + uintptr_t(L.total)};
     const Range rx{uintptr_t(X), uintptr_t(X) + uintptr_t(M * K * 2)};
-    const Range ry{uintptr_t(Y), uintptr_t(Y) + uintptr_t(M * N * 4)};
+    const Range ry{uintptr_t(Y), uintptr_t(Y) + uintptr_t(y_bytes(epi, M, N))};
     if (overlap(ry, rw) || overlap(ry, rx)) return EMB_EINVAL;
     return EMB_OK;
 }
 
-MatRef mat_ref(int fmt, const void* W, float* Y, int64_t N, int64_t K) {
+MatRef mat_ref(int fmt, const void* W, void* Y, int64_t N, int64_t K) {
     const Layout L = layout_of(fmt, N, K);
     const uint8_t* base = static_cast<const uint8_t*>(W);
     return MatRef{base, reinterpret_cast<const __half*>(base + L.scales_off), Y, N,
@@ -139,10 +149,11 @@ emb_status emb_quantize_q6_0(const float* W, int64_t N, int64_t K, void* W_block
 
 emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_t* X, float* Y, int64_t M,
                        int64_t N, int64_t K, emb_stream_t stream) {
-    const emb_status st = check_layer(fmt, W_blocks, X, Y, M, N, K);
+    const emb_status st = check_layer(fmt, EMB_EPI_F32, W_blocks, X, Y, M, N, K);
     if (st != EMB_OK) return st;
     GroupRef g = {};
     g.fmt = fmt;
+    g.epi = EMB_EPI_F32;
     g.n_mats = 1;
     g.mats[0] = mat_ref(fmt, W_blocks, Y, N, K);
     g.X = reinterpret_cast<const __nv_bfloat16*>(X);
@@ -153,13 +164,15 @@ emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_t* X, fl
     return from_cuda(launch_group(g, false, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-// Group consecutive layers that read the same X with the same format and K, when no
-// member's Y overlaps another member's W or Y (they then run in one launch).
+static Range y_range_of(const emb_qlayer& L, int64_t M) {
+    return Range{uintptr_t(L.Y), uintptr_t(L.Y) + uintptr_t(y_bytes(L.epilogue, M, L.N))};
+}
+
+// Group consecutive layers that read the same X with the same format, K and epilogue,
+// when no member's Y overlaps another member's W or Y (they then run in one launch).
 static std::vector<std::pair<int, int>> plan_groups(const emb_qlayer* layers, int n, int64_t M) {
     std::vector<std::pair<int, int>> groups;  // [first, last)
-    auto y_range = [&](int b) {
-        return Range{uintptr_t(layers[b].Y), uintptr_t(layers[b].Y) + uintptr_t(M * layers[b].N * 4)};
-    };
+    auto y_range = [&](int b) { return y_range_of(layers[b], M); };
     auto w_range = [&](int a) {
         const Layout La = layout_of(layers[a].fmt, layers[a].N, layers[a].K);
         return Range{uintptr_t(layers[a].W_blocks), uintptr_t(layers[a].W_blocks) + uintptr_t(La.total)};
@@ -168,7 +181,8 @@ static std::vector<std::pair<int, int>> plan_groups(const emb_qlayer* layers, in
     while (i < n) {
         int j = i + 1;
         while (j < n && j - i < kMaxGroup && layers[j].X == layers[i].X &&
-               layers[j].fmt == layers[i].fmt && layers[j].K == layers[i].K) {
+               layers[j].fmt == layers[i].fmt && layers[j].K == layers[i].K &&
+               layers[j].epilogue == layers[i].epilogue) {
             bool clash = false;
             for (int a = i; a <= j && !clash; ++a)
                 for (int b = i; b <= j && !clash; ++b)
@@ -187,20 +201,18 @@ static emb_status check_seq(const emb_qlayer* layers, int n_layers, int64_t M) {
     if (!layers || n_layers < 1 || n_layers > EMB_MAX_LAYERS || M < 1) return EMB_EINVAL;
     for (int j = 0; j < n_layers; ++j) {
         const emb_qlayer& L = layers[j];
-        if (L.reserved != 0) return EMB_EINVAL;
-        const emb_status st = check_layer(L.fmt, L.W_blocks, L.X, L.Y, M, L.N, L.K);
+        const emb_status st = check_layer(L.fmt, L.epilogue, L.W_blocks, L.X, L.Y, M, L.N, L.K);
         if (st != EMB_OK) return st;
     }
-    // a layer's inputs (X, W) may not be written by the same or an earlier layer
+    // a layer's weights may not be written by the same or an earlier layer: every launch
+    // fetches its weights before waiting for the previous one. X may be an earlier layer's
+    // output (read after that layer's launch has completed).
     for (int j = 0; j < n_layers; ++j) {
         const emb_qlayer& Lj = layers[j];
-        const Range xj{uintptr_t(Lj.X), uintptr_t(Lj.X) + uintptr_t(M * Lj.K * 2)};
         const Range wj{uintptr_t(Lj.W_blocks),
                        uintptr_t(Lj.W_blocks) + uintptr_t(layout_of(Lj.fmt, Lj.N, Lj.K).total)};
-        for (int i = 0; i < j; ++i) {
-            const Range yi{uintptr_t(layers[i].Y), uintptr_t(layers[i].Y) + uintptr_t(M * layers[i].N * 4)};
-            if (overlap(yi, xj) || overlap(yi, wj)) return EMB_EINVAL;
-        }
+        for (int i = 0; i < j; ++i)
+            if (overlap(y_range_of(layers[i], M), wj)) return EMB_EINVAL;
     }
     return EMB_OK;
 }
@@ -222,6 +234,7 @@ static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
         const emb_qlayer& L0 = layers[gr.first];
         GroupRef g = {};
         g.fmt = L0.fmt;
+        g.epi = L0.epilogue;
         g.n_mats = gr.second - gr.first;
         for (int k = 0; k < g.n_mats; ++k) {
             const emb_qlayer& L = layers[gr.first + k];

@@ -33,6 +33,34 @@ __host__ __device__ inline Layout layout_of(int fmt, int64_t N, int64_t K) {
     return L;
 }
 
+// ------------------------------------------------------------------ epilogues
+// Activations of the gated epilogues, in fp32 with the CUDA math library.
+__device__ __forceinline__ float act_gelu_tanh(float g) {
+    return 0.5f * g * (1.0f + tanhf(0.7978845608028654f * (g + 0.044715f * g * g * g)));
+}
+__device__ __forceinline__ float act_silu(float g) { return g / (1.0f + expf(-g)); }
+
+// Store one result v for element (m, n) of a Y with N columns.
+__device__ __forceinline__ void epi_store(int epi, void* Y, int64_t m, int64_t n, int64_t N, float v) {
+    const int64_t i = m * N + n;
+    if (epi == EMB_EPI_BF16) {
+        reinterpret_cast<__nv_bfloat16*>(Y)[i] = __float2bfloat16_rn(v);
+    } else if (epi == EMB_EPI_ADD) {
+        float* y = reinterpret_cast<float*>(Y);
+        y[i] = __fadd_rn(y[i], v);
+    } else {
+        reinterpret_cast<float*>(Y)[i] = v;
+    }
+}
+
+// Gated epilogues: gate row n (even) and up row n + 1 give element (m, n / 2) of a bf16 Y
+// with N / 2 columns.
+__device__ __forceinline__ void epi_store_gated(int epi, void* Y, int64_t m, int64_t n, int64_t N,
+                                                float gate, float up) {
+    const float a = (epi == EMB_EPI_GEGLU) ? act_gelu_tanh(gate) : act_silu(gate);
+    reinterpret_cast<__nv_bfloat16*>(Y)[m * (N / 2) + n / 2] = __float2bfloat16_rn(__fmul_rn(a, up));
+}
+
 // Device status word values (bit flags, OR-ed by kernels).
 constexpr int kStatusTimeout = 1;
 
@@ -58,13 +86,14 @@ constexpr int kMaxGroup = 4;
 struct MatRef {
     const uint8_t* codes;   // Q6_0: the low-nibble plane
     const __half* scales;
-    float* Y;
+    void* Y;                // as the group's epilogue says
     int64_t N;
     const uint8_t* high;    // Q6_0: the 2-bit high plane; else nullptr
 };
 
 struct GroupRef {
     int fmt;
+    int epi;                // emb_epilogue of every member
     int n_mats;
     MatRef mats[kMaxGroup];
     const __nv_bfloat16* X;

@@ -66,7 +66,7 @@ struct GemmParams {
     CUtensorMap codes_map[kMaxGroup];      // codes [N][row bytes] u8, box {128, 128}, 128B swizzle
     CUtensorMap scales_map[kMaxGroup];     // scales [N][ldS] u16, box {8, 128}
     CUtensorMap high_map[kMaxGroup];       // Q6_0 high bits [N][K/4] u8, box {64, 128}, no swizzle
-    float* Y[kMaxGroup];
+    void* Y[kMaxGroup];                    // as the epilogue says
     int32_t N[kMaxGroup];
     int32_t tile0[kMaxGroup + 1];
     int32_t n_mats;
@@ -74,6 +74,7 @@ struct GemmParams {
     int32_t T;                             // tokens per token tile, multiple of 16, <= 256
     int32_t P;                             // token tiles per CTA (1, or 2 sharing each A tile)
     int32_t splits;                        // K splits (cluster size along z)
+    int32_t epi;                           // emb_epilogue
     int32_t stages;                        // A/X ring depth
     int32_t a_gap0;                        // P = 2: TMEM column of the first A stage after tile 0's
     int32_t a_per_gap;                     //   accumulator, and A stages per gap (see pick_stages_pair)
@@ -456,17 +457,28 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16) + uint32_t(tt * kAccCols);
             const int n = n0 + row;
             const int mt = m0 + tt * T;  // first token of that tile
-            float* Y = p.Y[g];
+            void* Y = p.Y[g];
+            const int epi = p.epi;
             for (int c0 = cbeg; c0 < cend; c0 += 16) {
                 uint32_t v[16];
                 ptx::tmem_ld_16(taddr + uint32_t(c0), v);
                 ptx::tmem_ld_wait();
                 if (splits == 1) {
-                    if (n < N) {
+                    if (epi >= EMB_EPI_GEGLU) {
+                        // gate row n (even lane) and up row n + 1 (the next lane): rows past N
+                        // hold zeros (their weights were read as zeros), so every lane shuffles
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const float up = __shfl_down_sync(0xffffffffu, __uint_as_float(v[e]), 1);
+                            const int m = mt + c0 + e;
+                            if ((lane & 1) == 0 && n < N && m < M)
+                                epi_store_gated(epi, Y, m, n, N, __uint_as_float(v[e]), up);
+                        }
+                    } else if (n < N) {
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
                             const int m = mt + c0 + e;
-                            if (m < M) Y[int64_t(m) * N + n] = __uint_as_float(v[e]);
+                            if (m < M) epi_store(epi, Y, m, n, N, __uint_as_float(v[e]));
                         }
                     }
                 } else {
@@ -490,8 +502,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             // 16-byte coalesced stores to Y[m][n..n+3]
             const int rows = kBN / splits, r0 = split * rows, q4 = rows / 4;
             const uint32_t pbase = ptx::smem_u32(part);
-            float* Y = p.Y[g];
-            const bool vec = (N % 4) == 0;
+            void* Y = p.Y[g];
+            const int epi = p.epi;
+            const bool vec = (N % 4) == 0 && epi == EMB_EPI_F32;
             for (int w = threadIdx.x - 64; w < q4 * T; w += kThreads - 64) {
                 const int c = w / q4, row = r0 + 4 * (w - c * q4);
                 const int m = m0 + c, n = n0 + row;
@@ -502,14 +515,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
                 }
                 if (m < M) {
-                    float* dst = Y + int64_t(m) * N + n;
                     if (vec && n + 3 < N) {
-                        *reinterpret_cast<float4*>(dst) = acc;
+                        *reinterpret_cast<float4*>(reinterpret_cast<float*>(Y) + int64_t(m) * N + n) = acc;
+                    } else if (epi >= EMB_EPI_GEGLU) {  // rows n, n + 2 are gate rows (n % 4 == 0)
+                        if (n < N) epi_store_gated(epi, Y, m, n, N, acc.x, acc.y);
+                        if (n + 2 < N) epi_store_gated(epi, Y, m, n + 2, N, acc.z, acc.w);
                     } else {
-                        if (n < N) dst[0] = acc.x;
-                        if (n + 1 < N) dst[1] = acc.y;
-                        if (n + 2 < N) dst[2] = acc.z;
-                        if (n + 3 < N) dst[3] = acc.w;
+                        if (n < N) epi_store(epi, Y, m, n, N, acc.x);
+                        if (n + 1 < N) epi_store(epi, Y, m, n + 1, N, acc.y);
+                        if (n + 2 < N) epi_store(epi, Y, m, n + 2, N, acc.z);
+                        if (n + 3 < N) epi_store(epi, Y, m, n + 3, N, acc.w);
                     }
                 }
             }
@@ -762,6 +777,7 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.P = P;
     p.stages = S;
     p.splits = splits;
+    p.epi = g.epi;
     p.tmem_cols = kTmemCols;
     p.status = status;
     if (g.fmt == EMB_Q8_0)

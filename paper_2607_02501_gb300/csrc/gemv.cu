@@ -31,11 +31,12 @@ struct GemvParams {
     const uint8_t* codes[kMaxGroup];
     const uint8_t* high[kMaxGroup];  // Q6_0: 2-bit high plane of each matrix
     const __half* scales[kMaxGroup];
-    float* Y[kMaxGroup];
+    void* Y[kMaxGroup];              // as the epilogue says
     int32_t N[kMaxGroup];
     int32_t tile0[kMaxGroup + 1];  // first row tile of each matrix (prefix sums)
     int32_t n_mats;
     int32_t M, K, ldS, U;          // U = 16-byte code units per row
+    int32_t epi;                   // emb_epilogue (gated: R even, gate/up row pairs)
     const __nv_bfloat16* X;
 };
 
@@ -259,13 +260,26 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
             if (lane == 0) red[warp][r * MT + j] = v;
         }
     __syncthreads();
-    if (t < R * MT) {
+    if (p.epi >= EMB_EPI_GEGLU) {
+        // gate row row0 + 2i and up row row0 + 2i + 1 (R is even) give one output
+        if (t < (R / 2) * MT) {
+            const int i = t / MT, j = t % MT;
+            float gate = 0.0f, up = 0.0f;
+#pragma unroll
+            for (int w = 0; w < NWARP; ++w) {
+                gate += red[w][(2 * i) * MT + j];
+                up += red[w][(2 * i + 1) * MT + j];
+            }
+            const int n = row0 + 2 * i, m = m0 + j;
+            if (n < N && m < p.M) epi_store_gated(p.epi, p.Y[g], m, n, N, gate, up);
+        }
+    } else if (t < R * MT) {
         const int r = t / MT, j = t % MT;
         float v = 0.0f;
 #pragma unroll
         for (int w = 0; w < NWARP; ++w) v += red[w][t];
         const int n = row0 + r, m = m0 + j;
-        if (n < N && m < p.M) p.Y[g][int64_t(m) * N + n] = v;
+        if (n < N && m < p.M) epi_store(p.epi, p.Y[g], m, n, N, v);
     }
 }
 
@@ -335,12 +349,13 @@ struct StagedParams {
     const uint8_t* codes[kMaxGroup];
     const uint8_t* high[kMaxGroup];  // Q6_0: 2-bit high plane of each matrix
     const __half* scales[kMaxGroup];
-    float* Y[kMaxGroup];
+    void* Y[kMaxGroup];              // as the epilogue says
     int32_t N[kMaxGroup];
     int32_t tile0[kMaxGroup + 1];  // first tile of each matrix (prefix sums)
     int32_t n_mats;
     int32_t M, K, ldS, U;
     int32_t TR, WK;                // rows per tile, warps along K
+    int32_t epi;                   // emb_epilogue (gated: RW and TR even)
     const __nv_bfloat16* X;
     int* status;
 };
@@ -459,21 +474,39 @@ __global__ void __launch_bounds__(kStageThreads) gemv_staged_kernel(const __grid
             for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
             if (lane == i * MT + t) mine = v;
         }
+    const bool gated = p.epi >= EMB_EPI_GEGLU;
     if (WK == 1) {
+        // gated: the up row's sum sits MT lanes further on (RW is even)
+        const float up = __shfl_down_sync(0xffffffffu, mine, MT);
         if (lane < RW * MT) {
             const int r = r0 + lane / MT, t = lane % MT;
-            if (r < rows && t < mt) p.Y[g][int64_t(m0 + t) * N + row0 + r] = mine;
+            if (r < rows && t < mt) {
+                if (!gated) epi_store(p.epi, p.Y[g], m0 + t, row0 + r, N, mine);
+                else if ((r & 1) == 0) epi_store_gated(p.epi, p.Y[g], m0 + t, row0 + r, N, mine, up);
+            }
         }
         return;
     }
     if (lane < RW * MT) red[(wk * p.TR + r0 + lane / MT) * MT + lane % MT] = mine;
     __syncthreads();
     // add the K slices in slice order
+    if (gated) {
+        for (int e = threadIdx.x; e < (rows / 2) * MT; e += kStageThreads) {
+            const int i = e / MT, t = e % MT;
+            float gate = 0.0f, up = 0.0f;
+            for (int k = 0; k < WK; ++k) {
+                gate += red[(k * p.TR + 2 * i) * MT + t];
+                up += red[(k * p.TR + 2 * i + 1) * MT + t];
+            }
+            if (t < mt) epi_store_gated(p.epi, p.Y[g], m0 + t, row0 + 2 * i, N, gate, up);
+        }
+        return;
+    }
     for (int e = threadIdx.x; e < rows * MT; e += kStageThreads) {
         float v = 0.0f;
         for (int k = 0; k < WK; ++k) v += red[k * p.TR * MT + e];
         const int r = e / MT, t = e % MT;
-        if (t < mt) p.Y[g][int64_t(m0 + t) * N + row0 + r] = v;
+        if (t < mt) epi_store(p.epi, p.Y[g], m0 + t, row0 + r, N, v);
     }
 }
 
@@ -516,7 +549,7 @@ cudaError_t launch_staged_rw(const StagedParams& p, int RW, int tiles, size_t sm
 // 3-6% (a shorter CTA lifetime shortens each launch's tail), e.g. Q8_0 32768 x 2048:
 // 14.9 us (8 rows) vs 15.8 us (16 rows); at M = 4, 32 KB tiles win (22.7 vs 27.0 us).
 bool pick_stage_shape(int fmt, int64_t rows_total, int64_t row_bytes, int U, int64_t tile_bytes,
-                      int& RW, int& WK) {
+                      bool even_rows, int& RW, int& WK) {
     static const int kQ8[5][2] = {{4, 1}, {4, 2}, {4, 4}, {2, 4}, {1, 4}};
     static const int kQ4[7][2] = {{4, 1}, {2, 1}, {1, 1}, {4, 2}, {4, 4}, {2, 4}, {1, 4}};
     const int n = (fmt == EMB_Q8_0) ? 5 : 7;
@@ -527,6 +560,7 @@ bool pick_stage_shape(int fmt, int64_t rows_total, int64_t row_bytes, int U, int
         const int64_t tr = int64_t(rw) * kStageWarps / wk;
         if (tr * row_bytes > tile_bytes) continue;
         if (wk > 1 && U / wk < 32) continue;
+        if (even_rows && (rw & 1)) continue;  // gated epilogues pair rows inside a warp
         RW = rw;
         WK = wk;
         found = true;
@@ -562,7 +596,8 @@ bool launch_staged(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     if (g.M == 1 && weight_row_bytes > kStageMaxRowBytesM1) return false;
     int RW = 0, WK = 0;
     const int64_t tile_bytes = (g.M == 1) ? kStageBytes / 2 : kStageBytes;
-    if (!pick_stage_shape(g.fmt, rows, weight_row_bytes, U, tile_bytes, RW, WK)) return false;
+    if (!pick_stage_shape(g.fmt, rows, weight_row_bytes, U, tile_bytes, g.epi >= EMB_EPI_GEGLU, RW, WK))
+        return false;
     StagedParams p = {};
     const int TR = RW * kStageWarps / WK;
     int tiles = 0;
@@ -583,6 +618,7 @@ bool launch_staged(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     p.U = U;
     p.TR = TR;
     p.WK = WK;
+    p.epi = g.epi;
     p.X = g.X;
     p.status = status;
     const size_t smem = kStageHeader + size_t(MT) * g.K * 2 + size_t(TR) * size_t(weight_row_bytes + g.ldS * 2);
@@ -633,13 +669,14 @@ constexpr int kMmaHeader = 128 + 512 * 4;  // barriers, then cross-warp sums [WK
 struct MmaParams {
     const uint8_t* codes[kMaxGroup];
     const __half* scales[kMaxGroup];
-    float* Y[kMaxGroup];
+    void* Y[kMaxGroup];              // as the epilogue says
     int32_t N[kMaxGroup];
     int32_t tile0[kMaxGroup + 1];
     int32_t n_mats;
     int32_t M, K, ldS;
     int32_t TR, WK;                // rows per tile (multiple of 16), warps along K
     int32_t pitch, spitch;         // padded shared-memory row pitch of codes / scales, bytes
+    int32_t epi;                   // emb_epilogue (element-wise kinds only)
     const __nv_bfloat16* X;
     int* status;
 };
@@ -753,15 +790,15 @@ __global__ void __launch_bounds__(kMmaThreads) gemv_q4_mma_kernel(const __grid_c
     }
     // acc[0], acc[1]: row gq, tokens 2t, 2t+1; acc[2], acc[3]: row gq + 8, same tokens
     const int ra = rg * 16 + gq, rb = ra + 8, m0 = 2 * t;
-    float* Yg = p.Y[g_mat];
+    void* Yg = p.Y[g_mat];
     if (WK == 1) {
         if (m0 < p.M) {
-            if (ra < rows) Yg[int64_t(m0) * N + row0 + ra] = acc[0];
-            if (rb < rows) Yg[int64_t(m0) * N + row0 + rb] = acc[2];
+            if (ra < rows) epi_store(p.epi, Yg, m0, row0 + ra, N, acc[0]);
+            if (rb < rows) epi_store(p.epi, Yg, m0, row0 + rb, N, acc[2]);
         }
         if (m0 + 1 < p.M) {
-            if (ra < rows) Yg[int64_t(m0 + 1) * N + row0 + ra] = acc[1];
-            if (rb < rows) Yg[int64_t(m0 + 1) * N + row0 + rb] = acc[3];
+            if (ra < rows) epi_store(p.epi, Yg, m0 + 1, row0 + ra, N, acc[1]);
+            if (rb < rows) epi_store(p.epi, Yg, m0 + 1, row0 + rb, N, acc[3]);
         }
         return;
     }
@@ -776,7 +813,7 @@ __global__ void __launch_bounds__(kMmaThreads) gemv_q4_mma_kernel(const __grid_c
         const int r = e / p.M, m = e % p.M;
         float v = 0.0f;
         for (int k = 0; k < WK; ++k) v += red[(k * p.TR + r) * 8 + m];
-        Yg[int64_t(m) * N + row0 + r] = v;
+        epi_store(p.epi, Yg, m, row0 + r, N, v);
     }
 }
 
@@ -787,7 +824,7 @@ __global__ void __launch_bounds__(kMmaThreads) gemv_q4_mma_kernel(const __grid_c
 // TR = 32 rows (2 row groups x 2 K slices) when that still gives 4 tiles per SM, else
 // 16 rows (4 K slices).
 bool launch_q4_mma(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
-    if (g.fmt != EMB_Q4_0 || g.M < 2 || g.M > kMmaMaxM) return false;
+    if (g.fmt != EMB_Q4_0 || g.M < 2 || g.M > kMmaMaxM || g.epi >= EMB_EPI_GEGLU) return false;
     const int64_t row_bytes = g.K / 2;
     if (row_bytes * 16 > kMmaTileBytes) return false;
     if (g.M * g.K * 2 > kStageXBytes) return false;
@@ -818,6 +855,7 @@ bool launch_q4_mma(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     p.WK = WK;
     p.pitch = int32_t(row_bytes + 16);
     p.spitch = int32_t(g.ldS * 2 + 16);
+    p.epi = g.epi;
     p.X = g.X;
     p.status = status;
     const size_t smem = size_t(kMmaHeader) + size_t(g.M) * g.K * 2 + size_t(TR) * (p.pitch + p.spitch);
@@ -859,7 +897,8 @@ cudaError_t launch_gemv_regs(const GroupRef& g, bool pdl, cudaStream_t s) {
     // rows per CTA: 4 (activation reuse across rows) unless that leaves the GPU idle;
     // 2 for long rows (U >= 320), where 4 rows leave too few CTAs per SM (measured on
     // GB300, M=1: Q8_0 2048 x 16384 10.8 us with 4 rows, 9.6 us with 2)
-    const int R = (rows < 4 * 2 * 152) ? 1 : (U >= 320) ? 2 : 4;
+    int R = (rows < 4 * 2 * 152) ? 1 : (U >= 320) ? 2 : 4;
+    if (g.epi >= EMB_EPI_GEGLU && R == 1) R = 2;  // gate/up row pairs inside one CTA
     int tiles = 0;
     for (int i = 0; i < g.n_mats; ++i) {
         p.codes[i] = g.mats[i].codes;
@@ -876,6 +915,7 @@ cudaError_t launch_gemv_regs(const GroupRef& g, bool pdl, cudaStream_t s) {
     p.K = int32_t(g.K);
     p.ldS = int32_t(g.ldS);
     p.U = U;
+    p.epi = g.epi;
     p.X = g.X;
     const int NT = pick_threads(U, g.fmt, tiles);
     const int M = int(g.M);

@@ -112,11 +112,12 @@ def test_seq_rejects(L):
     assert L.emb_qlayer_seq(arr, emb.EMB_MAX_LAYERS + 1, M, None, 0, None) == emb.EMB_EINVAL
     assert L.emb_qlayer_seq(arr, 1, 0, None, 0, None) == emb.EMB_EINVAL
     bad = _layers([good])
-    bad[0].reserved = 1
+    bad[0].epilogue = 5                                    # unknown epilogue
     assert L.emb_qlayer_seq(bad, 1, M, None, 0, None) == emb.EMB_EINVAL
-    # layer 1 reads (as X) what layer 0 writes
-    chain = _layers([good, (0, A + (64 << 20), 128, 64, C, C + (1 << 20))])
-    assert L.emb_qlayer_seq(chain, 2, M, None, 0, None) == emb.EMB_EINVAL
+    bad[0].epilogue = -1
+    assert L.emb_qlayer_seq(bad, 1, M, None, 0, None) == emb.EMB_EINVAL
+    odd = _layers([(0, A, 127, 64, B, C, emb.EMB_EPI_GEGLU)])   # gated needs even N
+    assert L.emb_qlayer_seq(odd, 1, M, None, 0, None) == emb.EMB_EINVAL
     # layer 1's weights overlap layer 0's output
     chain = _layers([good, (0, C, 128, 64, B, C + (1 << 20))])
     assert L.emb_qlayer_seq(chain, 2, M, None, 0, None) == emb.EMB_EINVAL
@@ -124,6 +125,25 @@ def test_seq_rejects(L):
     chain = _layers([good, (1, A + (64 << 20), 128, 64, B + 8, C + (1 << 20))])
     assert L.emb_qlayer_seq(chain, 2, M, None, 0, None) == emb.EMB_EALIGN
     assert L.emb_qlayer_seq_workspace(chain, 2, M) == ctypes.c_size_t(-1).value
+
+
+def test_seq_epilogue_overlap_rules(L):
+    """A layer may read (as X) an earlier layer's output; weights may not be written;
+    Y's extent follows the epilogue (bf16: 2 bytes per element, gated: N/2 columns)."""
+    M = 1
+    # layer 1 reads layer 0's bf16 output as its X: accepted (no launch on the CPU: the
+    # checks pass and the call then needs a GPU, so use the workspace query to validate)
+    chain = _layers([(0, A, 128, 64, B, C, emb.EMB_EPI_BF16),
+                     (0, A + (64 << 20), 128, 128, C, C + (1 << 20))])
+    assert emb.emb_qlayer_seq_workspace(chain, M) == 0
+    # layer 1's weights overlap layer 0's output: rejected
+    chain = _layers([(0, A, 128, 64, B, C, emb.EMB_EPI_BF16), (0, C, 128, 64, B, C + (1 << 20))])
+    assert L.emb_qlayer_seq_workspace(chain, 2, M) == ctypes.c_size_t(-1).value
+    # a gated layer writes M x N/2 bf16: 64 x 2 = 128 bytes, so X right behind is fine
+    ok = _layers([(0, A, 128, 64, C + 128, C, emb.EMB_EPI_GEGLU)])
+    assert emb.emb_qlayer_seq_workspace(ok, M) == 0
+    bad = _layers([(0, A, 128, 64, C + 64, C, emb.EMB_EPI_GEGLU)])   # X inside Y
+    assert L.emb_qlayer_seq_workspace(bad, 1, M) == ctypes.c_size_t(-1).value
 
 
 def test_seq_workspace_is_zero_for_valid_chains(L):
@@ -142,8 +162,10 @@ def test_chain_create_rejects(L):
     assert L.emb_chain_create(None, 1, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
     assert h.value is None   # cleared on failure
     assert L.emb_chain_create(arr, 0, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
-    chain = _layers([good, (0, A + (64 << 20), 128, 64, C, C + (1 << 20))])   # reads layer 0's Y
+    chain = _layers([good, (0, C, 128, 64, B, C + (1 << 20))])   # weights are layer 0's Y
     assert L.emb_chain_create(chain, 2, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
+    odd = _layers([(0, A, 127, 64, B, C, emb.EMB_EPI_SWIGLU)])      # gated with odd N
+    assert L.emb_chain_create(odd, 1, M, None, 0, ctypes.byref(h)) == emb.EMB_EINVAL
     chain = _layers([good, (1, A + (64 << 20), 128, 64, B + 8, C + (1 << 20))])   # misaligned X
     assert L.emb_chain_create(chain, 2, M, None, 0, ctypes.byref(h)) == emb.EMB_EALIGN
     assert L.emb_chain_launch(None, None) == emb.EMB_EINVAL
