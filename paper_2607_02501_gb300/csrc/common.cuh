@@ -61,6 +61,32 @@ __device__ __forceinline__ void epi_store_gated(int epi, void* Y, int64_t m, int
     reinterpret_cast<__nv_bfloat16*>(Y)[m * (N / 2) + n / 2] = __float2bfloat16_rn(__fmul_rn(a, up));
 }
 
+// Results v of elements (m, n .. n + 3), N % 4 == 0 and n % 4 == 0 (Y 16-byte aligned): one
+// 16-byte (fp32, residual add), 8-byte (bf16) or 4-byte (gated: gate rows n, n + 2, up rows
+// n + 1, n + 3) access, with the same roundings as epi_store / epi_store_gated.
+__device__ __forceinline__ void epi_store4(int epi, void* Y, int64_t m, int64_t n, int64_t N, float4 v) {
+    const int64_t i = m * N + n;
+    if (epi == EMB_EPI_F32) {
+        *reinterpret_cast<float4*>(reinterpret_cast<float*>(Y) + i) = v;
+    } else if (epi == EMB_EPI_ADD) {
+        float4* y = reinterpret_cast<float4*>(reinterpret_cast<float*>(Y) + i);
+        const float4 o = *y;
+        *y = make_float4(__fadd_rn(o.x, v.x), __fadd_rn(o.y, v.y), __fadd_rn(o.z, v.z),
+                         __fadd_rn(o.w, v.w));
+    } else if (epi == EMB_EPI_BF16) {
+        const __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+        uint2 u;
+        u.x = *reinterpret_cast<const uint32_t*>(&lo);
+        u.y = *reinterpret_cast<const uint32_t*>(&hi);
+        *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(Y) + i) = u;
+    } else {
+        const float a0 = (epi == EMB_EPI_GEGLU) ? act_gelu_tanh(v.x) : act_silu(v.x);
+        const float a1 = (epi == EMB_EPI_GEGLU) ? act_gelu_tanh(v.z) : act_silu(v.z);
+        *reinterpret_cast<__nv_bfloat162*>(reinterpret_cast<__nv_bfloat16*>(Y) + m * (N / 2) + n / 2) =
+            __floats2bfloat162_rn(__fmul_rn(a0, v.y), __fmul_rn(a1, v.w));
+    }
+}
+
 // Device status word values (bit flags, OR-ed by kernels).
 constexpr int kStatusTimeout = 1;
 

@@ -474,6 +474,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                             if ((lane & 1) == 0 && n < N && m < M)
                                 epi_store_gated(epi, Y, m, n, N, __uint_as_float(v[e]), up);
                         }
+                    } else if (epi == EMB_EPI_ADD && n < N) {
+                        // reads four at a time ahead of their stores: a read after a store to
+                        // the same buffer would otherwise wait for that store
+                        float* y = reinterpret_cast<float*>(Y);
+#pragma unroll
+                        for (int e0 = 0; e0 < 16; e0 += 4) {
+                            float old[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                old[e] = (mt + c0 + e0 + e < M) ? y[int64_t(mt + c0 + e0 + e) * N + n] : 0.0f;
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                if (mt + c0 + e0 + e < M)
+                                    y[int64_t(mt + c0 + e0 + e) * N + n] =
+                                        __fadd_rn(old[e], __uint_as_float(v[e0 + e]));
+                        }
                     } else if (n < N) {
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
@@ -504,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint32_t pbase = ptx::smem_u32(part);
             void* Y = p.Y[g];
             const int epi = p.epi;
-            const bool vec = (N % 4) == 0 && epi == EMB_EPI_F32;
+            const bool vec = (N % 4) == 0;
             for (int w = threadIdx.x - 64; w < q4 * T; w += kThreads - 64) {
                 const int c = w / q4, row = r0 + 4 * (w - c * q4);
                 const int m = m0 + c, n = n0 + row;
@@ -516,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 }
                 if (m < M) {
                     if (vec && n + 3 < N) {
-                        *reinterpret_cast<float4*>(reinterpret_cast<float*>(Y) + int64_t(m) * N + n) = acc;
+                        epi_store4(epi, Y, m, n, N, acc);
                     } else if (epi >= EMB_EPI_GEGLU) {  // rows n, n + 2 are gate rows (n % 4 == 0)
                         if (n < N) epi_store_gated(epi, Y, m, n, N, acc.x, acc.y);
                         if (n + 2 < N) epi_store_gated(epi, Y, m, n + 2, N, acc.z, acc.w);

@@ -25,6 +25,17 @@ FMT_NAMES = {Q8_0: "Q8_0", Q4_0: "Q4_0", Q6_0: "Q6_0"}
 BLOCK_BYTES = {Q8_0: 34, Q4_0: 18, Q6_0: 26}   # packed bytes per 32 weights (codes + fp16 scale)
 
 
+# layer epilogues (the library's emb_epilogue values)
+EPI_F32, EPI_BF16, EPI_ADD, EPI_GEGLU, EPI_SWIGLU = 0, 1, 2, 3, 4
+
+
+def output_bytes(epilogue: int, M: int, N: int) -> int:
+    """Bytes a layer's output moves: fp32 write, bf16 write, fp32 read + write (residual
+    add), or one bf16 per gate/up row pair."""
+    return {EPI_F32: 4 * M * N, EPI_BF16: 2 * M * N, EPI_ADD: 8 * M * N,
+            EPI_GEGLU: M * N, EPI_SWIGLU: M * N}[epilogue]
+
+
 @dataclasses.dataclass(frozen=True)
 class Linear:
     """One weight matrix W [N][K] (PyTorch Linear.weight layout)."""
@@ -33,6 +44,9 @@ class Linear:
     K: int
     seed: int
     outliers: float = 0.0  # fraction of weights multiplied by 8 before quantisation
+    epilogue: int = EPI_F32
+    # the layer's X is the output of the group this many groups earlier (0: its own input)
+    x_from: int = 0
 
 
 @dataclasses.dataclass(frozen=True)
@@ -58,8 +72,9 @@ class Workload:
         return sum(l.N * l.K // 32 * per for l in self.linears())
 
     def algorithmic_bytes(self) -> int:
-        """Weights read once + X read once (bf16) + Y written once (fp32), per pass."""
-        return self.weight_bytes() + sum(self.M * l.K * 2 + self.M * l.N * 4
+        """Weights read once + X read once (bf16) + the output per the layer's epilogue
+        (fp32 written once unless fused), per pass."""
+        return self.weight_bytes() + sum(self.M * l.K * 2 + output_bytes(l.epilogue, self.M, l.N)
                                          for l in self.linears())
 
     def flops(self) -> int:
@@ -110,6 +125,26 @@ def action_expert_denoise() -> Workload:
     return Workload("action_expert_q8_0_m50_x10", Q8_0, 50, 18,
                     _flatten_layers(_decoder_layers("A", 18, 1024, 128, 4096, 3000)),
                     repeats=10)
+
+
+def action_expert_fused(steps: int = 10) -> Workload:
+    """The action expert's flow-matching loop as one chain: `steps` denoising steps x 18
+    layers, M = 50, Q8_0, with fused epilogues: q/k/v write bf16 (the attention's inputs),
+    o and down add into one fp32 residual stream, gate/up is one matrix of interleaved
+    rows whose GeGLU output (bf16) is down's input."""
+    groups = []
+    for step in range(steps):
+        for layer in range(18):
+            s = 3000 + 16 * layer      # the same weights every step
+            a = f"A{layer}"
+            groups.append([Linear(f"{a}.q", 1024, 1024, s + 0, epilogue=EPI_BF16),
+                           Linear(f"{a}.k", 128, 1024, s + 1, epilogue=EPI_BF16),
+                           Linear(f"{a}.v", 128, 1024, s + 2, epilogue=EPI_BF16)])
+            groups.append([Linear(f"{a}.o", 1024, 1024, s + 3, epilogue=EPI_ADD)])
+            groups.append([Linear(f"{a}.gate_up", 2 * 4096, 1024, s + 4, epilogue=EPI_GEGLU)])
+            groups.append([Linear(f"{a}.down", 1024, 4096, s + 6, epilogue=EPI_ADD, x_from=1)])
+    return Workload(f"action_expert_fused_q8_0_m50_x{steps}", Q8_0, 50, 18 * steps,
+                    _flatten_layers(groups))
 
 
 def gemma2b_prefill(fmt: int) -> Workload:
