@@ -268,3 +268,8 @@ def epilogue_reference(kind: int, Y, B, R=None):
     bound = (np.abs(act) * Bu + (np.abs(u) + Bu) * (1.2 * Bg + 2.0 ** -20 * (np.abs(g) + Bg + 1.0))
              + 2.0 ** -8 * np.abs(h) + 1e-6)
     return h, bound
+
+
+# The non-matmul steps of a backbone / action-expert layer (RMSNorm, rotary embedding,
+# attention): oracle/layer.py.
+from .layer import attention_reference, rmsnorm_reference, rope_reference  # noqa: E402,F401
