@@ -47,9 +47,12 @@ def rope_reference(x, n_heads: int, head_dim: int, pos0: int, base: float):
     """x: bf16 values as floats [M][n_heads * head_dim], token m at position pos0 + m.
     Returns (ref, bound) of the same shape.
 
-    Bound: the kernel forms each angle and its cosine and sine in fp64 (error far below
-    fp32's), then x_a cos - x_b sin (or x_b cos + x_a sin) in fp32: two products and one
-    add, at most 3 u (|x_a| + |x_b|); the bf16 store adds 2^-8 of the value."""
+    Bound: the kernel forms each angle as an exact two-float product of the position and
+    a two-float inverse frequency (error ~|angle| 2^-46), takes its cosine and sine with
+    fp32 sincosf (within 2 ulp) corrected to first order by the angle's low part, so each
+    is within 2^-21 of the exact value; then x_a cos - x_b sin (or x_b cos + x_a sin) in
+    fp32, two products and one add, at most 3 u (|x_a| + |x_b|) more; the bf16 store adds
+    2^-8 of the value."""
     x = np.asarray(x, dtype=np.float64)
     M = x.shape[0]
     half = head_dim // 2
@@ -67,7 +70,7 @@ def rope_reference(x, n_heads: int, head_dim: int, pos0: int, base: float):
         m = np.abs(a) + np.abs(b)
         mag[:, h * head_dim:h * head_dim + half] = m
         mag[:, h * head_dim + half:(h + 1) * head_dim] = m
-    e = 4 * U32 * mag
+    e = (2.0 ** -21 + 4 * U32) * mag
     bound = e + U_BF16 * (np.abs(ref) + e) + 1e-38
     return ref, bound
 
