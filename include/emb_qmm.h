@@ -206,6 +206,61 @@ EMB_API emb_status emb_chain_launch(emb_chain_t chain, emb_stream_t stream);
 /* Free the recording (NULL is a no-op). Replays already enqueued still complete. */
 EMB_API emb_status emb_chain_destroy(emb_chain_t chain);
 
+/* Record any sequence of this library's calls as one chain (graph replay of a whole layer
+ * or loop, Section 3.2 principle 2). After emb_chain_record_begin(stream), every library
+ * call made by this thread on `stream` is recorded instead of run (CUDA stream capture in
+ * thread-local mode) until emb_chain_record_end(stream, &chain) returns the recording,
+ * which emb_chain_launch replays and emb_chain_destroy frees. The recording holds every
+ * pointer the recorded calls were given; callers keep those buffers alive. Between begin
+ * and end no call may synchronise (emb_device_status) and arguments are validated as
+ * usual (an invalid call records nothing and returns its error; the recording goes on).
+ * stream: a created (non-NULL) stream of the current device.
+ * Errors: EMB_EINVAL (NULL stream or chain pointer), EMB_ECUDA (capture could not begin or
+ * end, or instantiation failed; *chain is then NULL). */
+EMB_API emb_status emb_chain_record_begin(emb_stream_t stream);
+EMB_API emb_status emb_chain_record_end(emb_stream_t stream, emb_chain_t* chain);
+
+/* ---------------------------------------------------------------- layer steps
+ * The steps of one transformer layer of the shared backbone and the action expert around
+ * its linears (the paper runs every model family through one backbone execution path,
+ * Section 3.2, and defines none of these operators; the standard definitions are used).
+ * All are enqueued on `stream` with programmatic dependent launch, like emb_qlayer_seq,
+ * allocate nothing, and are deterministic. bf16 buffers hold bit patterns (uint16_t). */
+
+/* RMSNorm (Zhang and Sennrich, 2019) of every token of the fp32 residual stream:
+ * y[m][i] = bf16(x[m][i] / sqrt(mean_i x[m][i]^2 + eps) * gamma[i]), the mean and square
+ * root in fp32 (correctly rounded square root and reciprocal), one bf16 rounding.
+ * x: device fp32 [M][D]; gamma: device fp32 [D]; y: device bf16 [M][D]; 16-byte aligned.
+ * 1 <= M < 2^31; D % 8 == 0, 8 <= D <= 65536; eps >= 0. y may not overlap x or gamma.
+ * Errors: EMB_EINVAL, EMB_EALIGN, EMB_ECUDA. */
+EMB_API emb_status emb_rmsnorm(const float* x, const float* gamma, uint16_t* y, int64_t M,
+                               int64_t D, float eps, emb_stream_t stream);
+
+/* Rotary position embedding (Su et al., 2021), rotate-half pairing, in place on bf16
+ * x [M][n_heads][head_dim]: token m sits at position pos0 + m; in every head, element i
+ * and element i + head_dim/2 (i < head_dim/2) are rotated by the angle
+ * (pos0 + m) * base^(-2i/head_dim): (a, b) -> (a cos - b sin, b cos + a sin). The
+ * inverse frequencies are formed in fp64 on the host, the angle as an exact two-float
+ * product, its cosine and sine in fp32 (error ~1e-7), the rotation in fp32, one bf16
+ * rounding. x: device, 16-byte aligned. head_dim even, 2..512; pos0 >= 0,
+ * pos0 + M <= 2^24 (positions exact in fp32); base > 0.
+ * Errors: EMB_EINVAL, EMB_EALIGN, EMB_ECUDA. */
+EMB_API emb_status emb_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim,
+                            int64_t pos0, float base, emb_stream_t stream);
+
+/* Scaled dot-product attention (Vaswani et al., 2017) of M query tokens over n0 + n1 keys:
+ * the prefix cache (K0, V0: [n0][n_kv_heads][head_dim]) followed by the chunk's own keys
+ * (K1, V1: [n1][n_kv_heads][head_dim]), all visible to every query (no mask). Query head h
+ * (Q: [M][n_heads][head_dim]) reads key/value head h / (n_heads / n_kv_heads);
+ * O[m][h] = sum_j softmax_j(scale * q.k_j) v_j, in fp32, one bf16 rounding.
+ * All bf16, device, 16-byte aligned; K0/V0 may be NULL when n0 == 0, K1/V1 when n1 == 0.
+ * n_heads % n_kv_heads == 0; head_dim 64 or 128 (else EMB_EUNSUPPORTED); n0 + n1 >= 1.
+ * O may not overlap any input. Errors: EMB_EINVAL, EMB_EALIGN, EMB_EUNSUPPORTED, EMB_ECUDA. */
+EMB_API emb_status emb_attention(const uint16_t* Q, const uint16_t* K0, const uint16_t* V0,
+                                 int64_t n0, const uint16_t* K1, const uint16_t* V1, int64_t n1,
+                                 uint16_t* O, int64_t M, int64_t n_heads, int64_t n_kv_heads,
+                                 int64_t head_dim, float scale, emb_stream_t stream);
+
 /* ---------------------------------------------------------------- test support
  * Dequantise W_blocks to fp32 [N][K] (w' exactly: the products are exact in fp32). */
 EMB_API emb_status emb_dequantize_f32(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,

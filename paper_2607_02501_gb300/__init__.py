@@ -103,6 +103,17 @@ def lib():
     L.emb_status_string.restype = ctypes.c_char_p
     L.emb_build_info.argtypes = []
     L.emb_build_info.restype = ctypes.c_char_p
+    L.emb_chain_record_begin.argtypes = [vp]
+    L.emb_chain_record_begin.restype = i32
+    L.emb_chain_record_end.argtypes = [vp, ctypes.POINTER(vp)]
+    L.emb_chain_record_end.restype = i32
+    f32 = ctypes.c_float
+    L.emb_rmsnorm.argtypes = [vp, vp, vp, i64, i64, f32, vp]
+    L.emb_rmsnorm.restype = i32
+    L.emb_rope.argtypes = [vp, i64, i64, i64, i64, f32, vp]
+    L.emb_rope.restype = i32
+    L.emb_attention.argtypes = [vp, vp, vp, i64, vp, vp, i64, vp, i64, i64, i64, i64, f32, vp]
+    L.emb_attention.restype = i32
     _lib = L
     return L
 
@@ -229,6 +240,76 @@ class RecordedChain:
             self.close()
         except Exception:
             pass
+
+
+def emb_chain_record_begin(stream) -> None:
+    _check(lib().emb_chain_record_begin(_stream(stream)), "emb_chain_record_begin")
+
+
+def emb_chain_record_end(stream) -> int:
+    h = ctypes.c_void_p()
+    _check(lib().emb_chain_record_end(_stream(stream), ctypes.byref(h)), "emb_chain_record_end")
+    return int(h.value)
+
+
+class Recording:
+    """Record library calls made on `stream` (a torch.cuda.Stream) inside the with-block
+    into one chain; `launch()` replays it, `close()` frees it. `keep` holds the buffers the
+    recording points at."""
+
+    def __init__(self, stream, keep=()):
+        self.stream = stream
+        self.keep = list(keep)
+        self.handle = 0
+
+    def __enter__(self):
+        emb_chain_record_begin(self.stream)
+        return self
+
+    def __exit__(self, exc_type, exc, tb):
+        h = emb_chain_record_end(self.stream)
+        if exc_type is None:
+            self.handle = h
+        elif h:
+            emb_chain_destroy(h)
+        return False
+
+    def launch(self, stream=None) -> None:
+        emb_chain_launch(self.handle, stream)
+
+    def close(self) -> None:
+        if self.handle:
+            emb_chain_destroy(self.handle)
+            self.handle = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def emb_rmsnorm(x, gamma, y, eps: float = 1e-6, stream=None) -> None:
+    """x: fp32 [M][D]; gamma: fp32 [D]; y: bf16 [M][D] (all device tensors)."""
+    M, D = x.shape
+    _check(lib().emb_rmsnorm(_ptr(x), _ptr(gamma), _ptr(y), M, D, eps, _stream(stream)), "emb_rmsnorm")
+
+
+def emb_rope(x, n_heads: int, head_dim: int, pos0: int, base: float = 10000.0, stream=None) -> None:
+    """In place on bf16 x [M][n_heads * head_dim]; token m at position pos0 + m."""
+    _check(lib().emb_rope(_ptr(x), x.shape[0], n_heads, head_dim, pos0, base, _stream(stream)),
+           "emb_rope")
+
+
+def emb_attention(Q, K0, V0, K1, V1, O, n_heads: int, n_kv_heads: int, head_dim: int,
+                  scale: float, stream=None) -> None:
+    """Q, O: bf16 [M][n_heads * head_dim]; K0/V0 (prefix) and K1/V1 (chunk): bf16
+    [n][n_kv_heads * head_dim] or None."""
+    n0 = 0 if K0 is None else K0.shape[0]
+    n1 = 0 if K1 is None else K1.shape[0]
+    _check(lib().emb_attention(_ptr(Q), _ptr(K0), _ptr(V0), n0, _ptr(K1), _ptr(V1), n1, _ptr(O),
+                               Q.shape[0], n_heads, n_kv_heads, head_dim, scale, _stream(stream)),
+           "emb_attention")
 
 
 def emb_dequantize_f32(fmt: int, W_blocks, N: int, K: int, out, stream=None) -> None:

@@ -15,7 +15,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libembqmm.so")
-SOURCES = ["api.cu", "quant.cu", "gemv.cu", "gemm_tc.cu"]
+SOURCES = ["api.cu", "quant.cu", "gemv.cu", "gemm_tc.cu", "layer_ops.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

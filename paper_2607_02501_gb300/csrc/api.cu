@@ -7,6 +7,7 @@
 // chain (the paper's latency-first fused execution, Section 3.2, design principle 2),
 // and the device status word that bounded device-side waits report into.
 #include <algorithm>
+#include <cmath>
 #include <mutex>
 #include <vector>
 
@@ -326,6 +327,77 @@ emb_status emb_chain_destroy(emb_chain_t chain) {
     return from_cuda(e);
 }
 
+emb_status emb_chain_record_begin(emb_stream_t stream) {
+    if (!stream) return EMB_EINVAL;  // the legacy default stream cannot be recorded
+    return from_cuda(cudaStreamBeginCapture(reinterpret_cast<cudaStream_t>(stream),
+                                            cudaStreamCaptureModeThreadLocal));
+}
+
+emb_status emb_chain_record_end(emb_stream_t stream, emb_chain_t* chain) {
+    if (!stream || !chain) return EMB_EINVAL;
+    *chain = nullptr;
+    cudaGraph_t graph = nullptr;
+    if (cudaStreamEndCapture(reinterpret_cast<cudaStream_t>(stream), &graph) != cudaSuccess || !graph) {
+        if (graph) cudaGraphDestroy(graph);
+        return EMB_ECUDA;
+    }
+    cudaGraphExec_t exec = nullptr;
+    const cudaError_t e = cudaGraphInstantiate(&exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) return EMB_ECUDA;
+    *chain = new emb_chain_st{exec};
+    return EMB_OK;
+}
+
+emb_status emb_rmsnorm(const float* x, const float* gamma, uint16_t* y, int64_t M, int64_t D,
+                       float eps, emb_stream_t stream) {
+    if (!x || !gamma || !y || M < 1 || M >= (int64_t(1) << 31) || D < 8 || D % 8 != 0 ||
+        D > 65536 || !(eps >= 0.0f) || !std::isfinite(eps))
+        return EMB_EINVAL;
+    if (!aligned(x, 16) || !aligned(gamma, 16) || !aligned(y, 16)) return EMB_EALIGN;
+    const Range ry{uintptr_t(y), uintptr_t(y) + uintptr_t(M * D * 2)};
+    if (overlap(ry, Range{uintptr_t(x), uintptr_t(x) + uintptr_t(M * D * 4)}) ||
+        overlap(ry, Range{uintptr_t(gamma), uintptr_t(gamma) + uintptr_t(D * 4)}))
+        return EMB_EINVAL;
+    return from_cuda(launch_rmsnorm(x, gamma, y, M, D, eps, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+emb_status emb_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim, int64_t pos0,
+                    float base, emb_stream_t stream) {
+    if (!x || M < 1 || n_heads < 1 || head_dim < 2 || head_dim % 2 != 0 || head_dim > 512 ||
+        pos0 < 0 || pos0 + M > (int64_t(1) << 24) || M * n_heads * head_dim >= (int64_t(1) << 46) ||
+        !(base > 0.0f) || !std::isfinite(base))
+        return EMB_EINVAL;
+    if (!aligned(x, 16)) return EMB_EALIGN;
+    return from_cuda(launch_rope(x, M, n_heads, head_dim, pos0, double(base),
+                                 reinterpret_cast<cudaStream_t>(stream)));
+}
+
+emb_status emb_attention(const uint16_t* Q, const uint16_t* K0, const uint16_t* V0, int64_t n0,
+                         const uint16_t* K1, const uint16_t* V1, int64_t n1, uint16_t* O, int64_t M,
+                         int64_t n_heads, int64_t n_kv_heads, int64_t head_dim, float scale,
+                         emb_stream_t stream) {
+    if (!Q || !O || M < 1 || M >= (int64_t(1) << 31) || n0 < 0 || n1 < 0 || n0 + n1 < 1 ||
+        n0 + n1 >= (int64_t(1) << 40) || n_heads < 1 || n_kv_heads < 1 || n_heads % n_kv_heads != 0 ||
+        n_heads > 4096 || !std::isfinite(scale))
+        return EMB_EINVAL;
+    if ((n0 > 0 && (!K0 || !V0)) || (n1 > 0 && (!K1 || !V1))) return EMB_EINVAL;
+    if (head_dim != 64 && head_dim != 128) return EMB_EUNSUPPORTED;
+    if (!aligned(Q, 16) || !aligned(O, 16) || (n0 > 0 && (!aligned(K0, 16) || !aligned(V0, 16))) ||
+        (n1 > 0 && (!aligned(K1, 16) || !aligned(V1, 16))))
+        return EMB_EALIGN;
+    const int64_t row = n_heads * head_dim * 2, kv_row = n_kv_heads * head_dim * 2;
+    const Range ro{uintptr_t(O), uintptr_t(O) + uintptr_t(M * row)};
+    if (overlap(ro, Range{uintptr_t(Q), uintptr_t(Q) + uintptr_t(M * row)})) return EMB_EINVAL;
+    const uint16_t* kv[4] = {K0, V0, K1, V1};
+    const int64_t cnt[4] = {n0, n0, n1, n1};
+    for (int i = 0; i < 4; ++i)
+        if (cnt[i] > 0 && overlap(ro, Range{uintptr_t(kv[i]), uintptr_t(kv[i]) + uintptr_t(cnt[i] * kv_row)}))
+            return EMB_EINVAL;
+    return from_cuda(launch_attention(Q, K0, V0, n0, K1, V1, n1, O, M, n_heads, n_kv_heads, head_dim,
+                                      scale, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 emb_status emb_dequantize_f32(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
                               float* out, emb_stream_t stream) {
     if (!valid_fmt(fmt) || !valid_shape(1, N, K) || !W_blocks || !out) return EMB_EINVAL;
@@ -373,9 +445,9 @@ const char* emb_status_string(emb_status status) {
 }
 
 const char* emb_build_info(void) {
-    return "libembqmm: sm_103a; Q8_0/Q4_0; GEMV (M<=4: staged/register FFMA2, Q4_0 mma.sync at M>=2) + "
+    return "libembqmm: sm_103a; Q8_0/Q6_0/Q4_0; GEMV (M<=4: staged/register FFMA2, Q4_0 mma.sync at M>=2) + "
            "tcgen05 GEMM (M>4: TMA, dequant to bf16 A tiles in TMEM, TMEM accumulators); "
-           "recorded chains (CUDA graphs)";
+           "recorded chains (CUDA graphs); RMSNorm, rotary embedding, grouped-head attention";
 }
 
 }  // extern "C"

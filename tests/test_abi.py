@@ -17,7 +17,7 @@ def L():
 
 def test_every_declared_symbol_is_exported(L):
     names = emb.declared_symbols()
-    assert len(names) == 16
+    assert len(names) == 21
     for n in names:
         assert hasattr(L, n), n
 
@@ -176,3 +176,60 @@ def test_library_has_no_torch_dependency():
     import subprocess
     out = subprocess.run(["ldd", emb.LIB_PATH], capture_output=True, text=True).stdout
     assert "torch" not in out and "libcudart" not in out
+
+
+D_ = C + (1 << 30)
+E_ = C + (2 << 30)
+
+
+def test_recording_rejects_null_stream_and_handle(L):
+    h = ctypes.c_void_p()
+    assert L.emb_chain_record_begin(None) == emb.EMB_EINVAL
+    assert L.emb_chain_record_end(None, ctypes.byref(h)) == emb.EMB_EINVAL
+    assert L.emb_chain_record_end(A, None) == emb.EMB_EINVAL
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((None, B, C, 4, 1024, 1e-6), emb.EMB_EINVAL),        # null x
+    ((A, B, C, 0, 1024, 1e-6), emb.EMB_EINVAL),           # M = 0
+    ((A, B, C, 4, 1028, 1e-6), emb.EMB_EINVAL),           # D % 8 != 0
+    ((A, B, C, 4, 1024, -1.0), emb.EMB_EINVAL),           # eps < 0
+    ((A, B, C, 4, 1024, float("nan")), emb.EMB_EINVAL),   # eps NaN
+    ((A + 4, B, C, 4, 1024, 1e-6), emb.EMB_EALIGN),       # x misaligned
+    ((A, B, C + 2, 4, 1024, 1e-6), emb.EMB_EALIGN),       # y misaligned
+    ((A, B, A + 4096, 4, 1024, 1e-6), emb.EMB_EINVAL),    # y inside x
+    ((A, B, B, 4, 1024, 1e-6), emb.EMB_EINVAL),           # y over gamma
+])
+def test_rmsnorm_validation(L, args, expect):
+    assert L.emb_rmsnorm(*args, None) == expect
+
+
+@pytest.mark.parametrize("args,expect", [
+    ((None, 50, 8, 128, 816, 1e4), emb.EMB_EINVAL),       # null x
+    ((A, 50, 8, 127, 816, 1e4), emb.EMB_EINVAL),          # odd head_dim
+    ((A, 50, 0, 128, 816, 1e4), emb.EMB_EINVAL),          # no heads
+    ((A, 50, 8, 128, -1, 1e4), emb.EMB_EINVAL),           # negative position
+    ((A, 50, 8, 128, 816, 0.0), emb.EMB_EINVAL),          # base <= 0
+    ((A, 50, 8, 1024, 816, 1e4), emb.EMB_EINVAL),         # head_dim > 512
+    ((A, 50, 8, 128, (1 << 24) - 10, 1e4), emb.EMB_EINVAL),  # positions past 2^24
+    ((A + 2, 50, 8, 128, 816, 1e4), emb.EMB_EALIGN),      # misaligned
+])
+def test_rope_validation(L, args, expect):
+    assert L.emb_rope(*args, None) == expect
+
+
+# Q, K0, V0, n0, K1, V1, n1, O, M, H, Hk, d, scale
+@pytest.mark.parametrize("args,expect", [
+    ((A, B, C, 816, D_, E_, 50, A + (3 << 20), 50, 8, 1, 96, 0.1), emb.EMB_EUNSUPPORTED),  # head_dim 96
+    ((A, B, C, 816, D_, E_, 50, A + (3 << 20), 50, 8, 3, 128, 0.1), emb.EMB_EINVAL),       # 8 % 3
+    ((A, B, C, 0, D_, E_, 0, A + (3 << 20), 50, 8, 1, 128, 0.1), emb.EMB_EINVAL),          # no keys
+    ((A, None, C, 816, D_, E_, 50, A + (3 << 20), 50, 8, 1, 128, 0.1), emb.EMB_EINVAL),    # K0 missing
+    ((A, B, C, 816, None, E_, 50, A + (3 << 20), 50, 8, 1, 128, 0.1), emb.EMB_EINVAL),     # K1 missing
+    ((A, B, C, 816, D_, E_, 50, A + 1024, 50, 8, 1, 128, 0.1), emb.EMB_EINVAL),            # O inside Q
+    ((A, B, C, 816, D_, E_, 50, B + 4096, 50, 8, 1, 128, 0.1), emb.EMB_EINVAL),            # O inside K0
+    ((A, B, C, 816, D_, E_, 50, A + (3 << 20), 50, 8, 1, 128, float("inf")), emb.EMB_EINVAL),
+    ((A, B + 8, C, 816, D_, E_, 50, A + (3 << 20), 50, 8, 1, 128, 0.1), emb.EMB_EALIGN),   # K0 misaligned
+])
+def test_attention_validation(L, args, expect):
+    assert L.emb_attention(*args, None) == expect
+
