@@ -80,14 +80,17 @@ def attention_reference(Q, K0, V0, K1, V1, n_heads: int, n_kv_heads: int, head_d
     """Q: [M][H*d]; K0, V0: [n0][Hk*d] (prefix cache); K1, V1: [n1][Hk*d] (the chunk's own
     keys and values); all bf16 values as floats. Returns (ref, bound), [M][H*d].
 
-    Bound, per query m and head h with n = n0 + n1 keys: each fp32 score carries an error
-    Delta <= (d + 2) u scale sum_i |q_i k_i| (exact bf16 products, d - 1 fp32 adds, the
-    scale); each exponential an error E <= 2^-21 + u |s_j - s_max| (expf within 2 ulp, plus
-    its argument's rounding), applied once per key block and once per rescale of the
-    running sums (at most n / 32 + 4 times). A relative perturbation rho = Delta + E (n / 32
-    + 4) of every unnormalised weight moves the normalised output by at most
-    2.2 rho sum_j p_j |v_j|; the fp32 sums of the weights and the weighted values add
-    2 (n + 8) u sum_j p_j |v_j|; the bf16 store adds 2^-8 |o|."""
+    Bound, per query m and head h with n = n0 + n1 keys. The kernel computes the scores and
+    the weighted values on tensor cores, whose fp32 accumulation need not round to nearest:
+    each addition is taken as an error of up to 2 u. So each score carries an error
+    Delta <= 2 (d + 2) u scale sum_i |q_i k_i| (exact bf16 products, d - 1 adds, the scale);
+    each exponential an error E <= 2^-21 + u |s_j - s_max| (expf within 2 ulp, plus its
+    argument's rounding), applied once per key block and once per rescale of the running
+    sums (at most n / 32 + 4 times); each weight enters the value product as a bf16 hi + lo
+    pair, within 2^-16 of it. A relative perturbation rho = Delta + E (n / 32 + 4) + 2^-16
+    of every unnormalised weight moves the normalised output by at most
+    2.2 rho sum_j p_j |v_j|; the sums of the weights and of the weighted values add
+    4 (n + 8) u sum_j p_j |v_j|; the bf16 store adds 2^-8 |o|."""
     Q = np.asarray(Q, dtype=np.float64)
     K = np.concatenate([np.asarray(K0, dtype=np.float64).reshape(-1, n_kv_heads * head_dim),
                         np.asarray(K1, dtype=np.float64).reshape(-1, n_kv_heads * head_dim)])
@@ -108,10 +111,10 @@ def attention_reference(Q, K0, V0, K1, V1, n_heads: int, n_kv_heads: int, head_d
         p = w / w.sum(axis=1, keepdims=True)
         o = p @ v                                                # [M][d]
         ref[:, h * head_dim:(h + 1) * head_dim] = o
-        delta = (head_dim + 2) * U32 * abs(scale) * (np.abs(q) @ np.abs(k).T).max(axis=1, keepdims=True)
+        delta = 2 * (head_dim + 2) * U32 * abs(scale) * (np.abs(q) @ np.abs(k).T).max(axis=1, keepdims=True)
         E = 2.0 ** -21 + U32 * (smax - s).max(axis=1, keepdims=True)
-        rho = delta + E * (n / 32.0 + 4.0)
+        rho = delta + E * (n / 32.0 + 4.0) + 2.0 ** -16
         spread = p @ np.abs(v)                                   # sum_j p_j |v_j|, [M][d]
-        b = (2.2 * rho + 2.0 * (n + 8) * U32) * spread
+        b = (2.2 * rho + 4.0 * (n + 8) * U32) * spread
         bound[:, h * head_dim:(h + 1) * head_dim] = b + U_BF16 * (np.abs(o) + b) + 1e-38
     return ref, bound
