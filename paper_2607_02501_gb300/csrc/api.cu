@@ -379,7 +379,7 @@ emb_status emb_attention(const uint16_t* Q, const uint16_t* K0, const uint16_t* 
                          emb_stream_t stream) {
     if (!Q || !O || M < 1 || M >= (int64_t(1) << 31) || n0 < 0 || n1 < 0 || n0 + n1 < 1 ||
         n0 + n1 >= (int64_t(1) << 40) || n_heads < 1 || n_kv_heads < 1 || n_heads % n_kv_heads != 0 ||
-        n_heads > 4096 || !std::isfinite(scale))
+        n_heads > 4096 || M * n_heads >= (int64_t(1) << 31) || !std::isfinite(scale))
         return EMB_EINVAL;
     if ((n0 > 0 && (!K0 || !V0)) || (n1 > 0 && (!K1 || !V1))) return EMB_EINVAL;
     if (head_dim != 64 && head_dim != 128) return EMB_EUNSUPPORTED;

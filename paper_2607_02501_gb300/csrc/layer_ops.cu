@@ -16,9 +16,6 @@
 namespace emb {
 namespace {
 
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
 cudaError_t launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t s,
                        void** args, unsigned cluster_z = 1) {
     cudaLaunchConfig_t cfg = {};
@@ -132,25 +129,29 @@ __global__ void __launch_bounds__(256) rope_kernel(const __grid_constant__ RopeP
 }
 
 // ------------------------------------------------------------------ attention
-// CTA = (query m, key/value head g with up to 8 of its query heads, key split z). Warp w
-// computes query head g * G + sub * 8 + w over this split's keys: key tiles of 64 staged
-// in shared memory by all 256 threads (bf16, key rows padded by one 32-bit word so that 32
-// lanes reading 32 different keys hit 32 banks), scores in fp32 (lane L scores keys L and
-// L + 32 of the tile), an online softmax per tile, and the weighted values accumulated in
-// fp32 (lane L owns D/32 consecutive dims). The splits of one (m, g, sub) form a cluster
-// along z; their (max, sum, output) triples are combined through distributed shared memory
-// in split order by the CTA whose rank matches the head (fixed order: deterministic).
-constexpr int kAttnWarps = 8;
+// Tensor-core attention (mma.sync m16n8k16, bf16 operands, fp32 accumulation). The rows of
+// one key/value head g are its (query m, head) pairs, row r = m * G + (h - g * G) with G the
+// heads per key/value head, so every query head of a group shares the key and value tiles.
+// CTA = (64 rows, key/value head, key split); warp w owns rows 16w..16w+15 of the CTA.
+// Per 64-key tile (double-buffered in shared memory by cp.async, rows padded by 16 bytes so
+// fragment loads are conflict-free): S = Q K^T (Q fragments held in registers for the whole
+// kernel), scale, an online softmax on the accumulator fragments (row max and sums over the
+// four lanes that share a row), then O += P V with P split into bf16 hi + lo parts (two MMAs,
+// weight error 2^-16) and V fragments from ldmatrix.trans. The key splits of one row block
+// form a cluster along z; their (max, sum, output) partials are combined through distributed
+// shared memory in split order (deterministic).
+constexpr int kAttnWarps = 4;
 constexpr int kAttnThreads = 32 * kAttnWarps;
+constexpr int kAttnRows = 16 * kAttnWarps;
 constexpr int kKeyTile = 64;
 
 template <int D>
 struct AttnSmem {
-    float q[kAttnWarps][D];
-    uint32_t k[kKeyTile][D / 2 + 1];  // bf16 pairs, one pad word per key row
-    uint32_t v[kKeyTile][D / 2];
-    float part_m[kAttnWarps], part_l[kAttnWarps];
-    float part_o[kAttnWarps][D];
+    static constexpr int kPitch = D + 8;                 // bf16 per padded key row
+    __nv_bfloat16 k[2][kKeyTile][kPitch];
+    __nv_bfloat16 v[2][kKeyTile][kPitch];
+    float part_o[kAttnRows][D];
+    float part_m[kAttnRows], part_l[kAttnRows];
 };
 
 struct AttnParams {
@@ -161,188 +162,274 @@ struct AttnParams {
     const __nv_bfloat16* V1;
     __nv_bfloat16* O;
     int64_t n0, n1;
-    int M, H, Hk, subgroups;  // subgroups: CTAs (of <= 8 heads) per key/value head
+    int M, H, Hk;
     float scale;
 };
 
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t saddr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                              uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(saddr));
+}
+
+// 16-byte global -> shared copy; src_bytes 0 writes zeros (the source is not read).
+__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(saddr), "l"(g), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+__device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+}
+
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __grid_constant__ AttnParams p) {
-    constexpr int DL = D / 32;  // dims per lane
-    static_assert(DL == 2 || DL == 4, "head_dim 64 or 128");
-    extern __shared__ __align__(16) uint8_t smem_raw[];
-    AttnSmem<D>& sm = *reinterpret_cast<AttnSmem<D>*>(smem_raw);
+    constexpr int KS = D / 16;  // k-steps of the score MMAs (head dims)
+    constexpr int NT = D / 8;   // n-tiles of the output (head dims)
+    using SM = AttnSmem<D>;
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    SM& sm = *reinterpret_cast<SM*>(smem_raw);
     ptx::griddep_launch_dependents();
     ptx::griddep_wait();  // Q and the chunk's keys and values come from the previous launches
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m = blockIdx.x;
-    const int g = blockIdx.y / p.subgroups, sub = blockIdx.y - g * p.subgroups;
-    const int G = p.H / p.Hk;
-    const int h0 = g * G + sub * kAttnWarps;
-    const int nh = min(kAttnWarps, G - sub * kAttnWarps);  // heads of this CTA
+    const int quad = lane >> 2, qc = lane & 3;
+    const int g = blockIdx.y, G = p.H / p.Hk;
+    const int64_t rows_total = int64_t(p.M) * G;
+    const int64_t row0 = int64_t(blockIdx.x) * kAttnRows;
     const int splits = gridDim.z, z = blockIdx.z;
     const int64_t n = p.n0 + p.n1;
     const int64_t k_lo = z * n / splits, k_hi = (z + 1) * n / splits;
     const int kv_stride = p.Hk * D;
 
-    // the CTA's queries, fp32
-    for (int e = threadIdx.x; e < nh * D; e += kAttnThreads) {
-        const int w = e / D, i = e - w * D;
-        sm.q[w][i] = __bfloat162float(p.Q[int64_t(m) * p.H * D + int64_t(h0 + w) * D + i]);
+    // global row -> (query, head) -> its Q / O row; nullptr past the last row
+    auto q_row = [&](int64_t r) -> int64_t {
+        return r < rows_total ? (r / G) * int64_t(p.H) * D + (int64_t(g) * G + r % G) * D : -1;
+    };
+    const int64_t rA = row0 + warp * 16 + quad, rB = rA + 8;
+    const int64_t offA = q_row(rA), offB = q_row(rB);
+
+    // Q fragments for the whole kernel (A operand, row-major 16 x D)
+    uint32_t qf[KS][4];
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks) {
+        const int c = ks * 16 + 2 * qc;
+        qf[ks][0] = offA >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offA + c) : 0u;
+        qf[ks][1] = offB >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offB + c) : 0u;
+        qf[ks][2] = offA >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offA + c + 8) : 0u;
+        qf[ks][3] = offB >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offB + c + 8) : 0u;
     }
 
-    float run_m = -INFINITY, run_l = 0.0f;
-    float acc[DL];
-#pragma unroll
-    for (int d = 0; d < DL; ++d) acc[d] = 0.0f;
-
-    // Key/value tiles: each thread moves kChunks 16-byte chunks of keys and of values per
-    // tile; the next tile's chunks are loaded into registers while this tile is computed.
-    constexpr int kChunks = kKeyTile * (D / 8) / kAttnThreads;
-    static_assert(kChunks * kAttnThreads == kKeyTile * (D / 8), "tile split");
-    uint4 kr[kChunks], vr[kChunks];
-    auto load_tile = [&](int64_t t0) {
-#pragma unroll
-        for (int u = 0; u < kChunks; ++u) {
-            const int e = threadIdx.x + u * kAttnThreads;
-            const int j = e / (D / 8), c = e - j * (D / 8);
+    // tile loader: 64 keys x D of keys and of values, 16-byte chunks, zero past the split
+    auto issue_tile = [&](int64_t t0, int stage) {
+        constexpr int kChunksPerRow = D / 8;
+        for (int e = threadIdx.x; e < kKeyTile * kChunksPerRow; e += kAttnThreads) {
+            const int j = e / kChunksPerRow, c = e - j * kChunksPerRow;
             const int64_t key = t0 + j;
-            if (key < k_hi) {
-                const __nv_bfloat16* kp = key < p.n0 ? p.K0 + key * kv_stride : p.K1 + (key - p.n0) * kv_stride;
-                const __nv_bfloat16* vp = key < p.n0 ? p.V0 + key * kv_stride : p.V1 + (key - p.n0) * kv_stride;
-                kr[u] = *reinterpret_cast<const uint4*>(kp + g * D + c * 8);
-                vr[u] = *reinterpret_cast<const uint4*>(vp + g * D + c * 8);
-            }
+            const bool ok = key < k_hi;
+            const int64_t kk = ok ? key : k_lo;  // any valid row when nothing is read
+            const __nv_bfloat16* kp = kk < p.n0 ? p.K0 + kk * kv_stride : p.K1 + (kk - p.n0) * kv_stride;
+            const __nv_bfloat16* vp = kk < p.n0 ? p.V0 + kk * kv_stride : p.V1 + (kk - p.n0) * kv_stride;
+            cp_async16(ptx::smem_u32(&sm.k[stage][j][c * 8]), kp + g * D + c * 8, ok ? 16 : 0);
+            cp_async16(ptx::smem_u32(&sm.v[stage][j][c * 8]), vp + g * D + c * 8, ok ? 16 : 0);
         }
     };
-    if (k_lo < k_hi) load_tile(k_lo);
-    for (int64_t t0 = k_lo; t0 < k_hi; t0 += kKeyTile) {
-        const int nt = int(k_hi - t0 < kKeyTile ? k_hi - t0 : int64_t(kKeyTile));
-        __syncthreads();  // the previous tile (and, first time, the queries) are consumed / written
+
+    float o[NT][4];
 #pragma unroll
-        for (int u = 0; u < kChunks; ++u) {
-            const int e = threadIdx.x + u * kAttnThreads;
-            const int j = e / (D / 8), c = e - j * (D / 8);
-            if (j < nt) {
-                sm.k[j][c * 4 + 0] = kr[u].x;
-                sm.k[j][c * 4 + 1] = kr[u].y;
-                sm.k[j][c * 4 + 2] = kr[u].z;
-                sm.k[j][c * 4 + 3] = kr[u].w;
-                *reinterpret_cast<uint4*>(&sm.v[j][c * 4]) = vr[u];
+    for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.0f;
+    float mA = -INFINITY, mB = -INFINITY, lA = 0.0f, lB = 0.0f;
+
+    const int ntiles = int((k_hi - k_lo + kKeyTile - 1) / kKeyTile);
+    if (ntiles > 0) issue_tile(k_lo, 0);
+    cp_async_commit();
+    for (int it = 0; it < ntiles; ++it) {
+        const int stage = it & 1;
+        const int64_t t0 = k_lo + int64_t(it) * kKeyTile;
+        if (it + 1 < ntiles) issue_tile(t0 + kKeyTile, stage ^ 1);
+        cp_async_commit();
+        cp_async_wait1();  // this thread's copies of tile `it` have landed
+        __syncthreads();   // and every thread's
+
+        // S = Q K^T for 64 keys: 8 n-tiles of 8 keys
+        float sc[8][4];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.0f;
+            const __nv_bfloat16* krow = &sm.k[stage][j * 8 + quad][0];
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                const uint32_t b0 = *reinterpret_cast<const uint32_t*>(krow + ks * 16 + 2 * qc);
+                const uint32_t b1 = *reinterpret_cast<const uint32_t*>(krow + ks * 16 + 2 * qc + 8);
+                mma_16816(sc[j], qf[ks], b0, b1);
             }
         }
-        __syncthreads();
-        if (t0 + kKeyTile < k_hi) load_tile(t0 + kKeyTile);
-        if (warp < nh) {
-            // scores of keys lane and lane + 32
-            float s0 = 0.0f, s1 = 0.0f;
-            const bool has0 = lane < nt, has1 = lane + 32 < nt;
-            const uint32_t* k0 = sm.k[has0 ? lane : 0];
-            const uint32_t* k1 = sm.k[has1 ? lane + 32 : 0];
-            const float* q = sm.q[warp];
-#pragma unroll 8
-            for (int i = 0; i < D / 2; ++i) {
-                const float2 qq = *reinterpret_cast<const float2*>(q + 2 * i);
-                const uint32_t a = k0[i], b = k1[i];
-                s0 = fmaf(qq.x, bf16_lo(a), s0);
-                s0 = fmaf(qq.y, bf16_hi(a), s0);
-                s1 = fmaf(qq.x, bf16_lo(b), s1);
-                s1 = fmaf(qq.y, bf16_hi(b), s1);
-            }
-            s0 = has0 ? __fmul_rn(s0, p.scale) : -INFINITY;
-            s1 = has1 ? __fmul_rn(s1, p.scale) : -INFINITY;
-            float tmax = fmaxf(s0, s1);
+        // scale, mask keys past the split, row maxima (rows A = quad, B = quad + 8)
+        float tA = -INFINITY, tB = -INFINITY;
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
-            const float new_m = fmaxf(run_m, tmax);  // finite: the tile has at least one key
-            const float corr = (run_m == -INFINITY) ? 0.0f : expf(run_m - new_m);
-            const float p0 = has0 ? expf(s0 - new_m) : 0.0f;
-            const float p1 = has1 ? expf(s1 - new_m) : 0.0f;
-            float psum = p0 + p1;
+        for (int j = 0; j < 8; ++j) {
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) psum += __shfl_xor_sync(0xffffffffu, psum, o);
-            run_l = run_l * corr + psum;
-            run_m = new_m;
-#pragma unroll
-            for (int d = 0; d < DL; ++d) acc[d] *= corr;
-            // weighted values: key j's weight comes from lane j % 32
-            for (int j = 0; j < nt; ++j) {
-                const float pj = __shfl_sync(0xffffffffu, j < 32 ? p0 : p1, j & 31);
-                if constexpr (DL == 4) {
-                    const uint2 vv = *reinterpret_cast<const uint2*>(&sm.v[j][lane * 2]);
-                    acc[0] = fmaf(pj, bf16_lo(vv.x), acc[0]);
-                    acc[1] = fmaf(pj, bf16_hi(vv.x), acc[1]);
-                    acc[2] = fmaf(pj, bf16_lo(vv.y), acc[2]);
-                    acc[3] = fmaf(pj, bf16_hi(vv.y), acc[3]);
-                } else {
-                    const uint32_t vv = sm.v[j][lane];
-                    acc[0] = fmaf(pj, bf16_lo(vv), acc[0]);
-                    acc[1] = fmaf(pj, bf16_hi(vv), acc[1]);
-                }
+            for (int e = 0; e < 2; ++e) {
+                const bool ok = t0 + j * 8 + 2 * qc + e < k_hi;
+                sc[j][e] = ok ? __fmul_rn(sc[j][e], p.scale) : -INFINITY;
+                sc[j][2 + e] = ok ? __fmul_rn(sc[j][2 + e], p.scale) : -INFINITY;
+                tA = fmaxf(tA, sc[j][e]);
+                tB = fmaxf(tB, sc[j][2 + e]);
             }
         }
+#pragma unroll
+        for (int x = 1; x <= 2; x <<= 1) {
+            tA = fmaxf(tA, __shfl_xor_sync(0xffffffffu, tA, x));
+            tB = fmaxf(tB, __shfl_xor_sync(0xffffffffu, tB, x));
+        }
+        const float nA = fmaxf(mA, tA), nB = fmaxf(mB, tB);  // finite: the tile has a key
+        const float cA = (mA == -INFINITY) ? 0.0f : expf(mA - nA);
+        const float cB = (mB == -INFINITY) ? 0.0f : expf(mB - nB);
+        mA = nA;
+        mB = nB;
+        float sA = 0.0f, sB = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                sc[j][e] = expf(sc[j][e] - nA);  // exp(-inf) = 0 for masked keys
+                sc[j][2 + e] = expf(sc[j][2 + e] - nB);
+                sA += sc[j][e];
+                sB += sc[j][2 + e];
+            }
+        }
+        lA = lA * cA + sA;  // lane-partial sums; the four lanes of a row are added at the end
+        lB = lB * cB + sB;
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+            o[j][0] *= cA;
+            o[j][1] *= cA;
+            o[j][2] *= cB;
+            o[j][3] *= cB;
+        }
+        // O += P V: 4 k-steps of 16 keys; P as hi + lo bf16 A fragments
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t ah[4], al[4];
+            const float* s0 = sc[2 * kk];
+            const float* s1 = sc[2 * kk + 1];
+            const float src[4][2] = {{s0[0], s0[1]}, {s0[2], s0[3]}, {s1[0], s1[1]}, {s1[2], s1[3]}};
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                ah[r] = pack_bf16x2(src[r][0], src[r][1]);
+                const float2 h = unpack_bf16x2(ah[r]);
+                al[r] = pack_bf16x2(__fsub_rn(src[r][0], h.x), __fsub_rn(src[r][1], h.y));
+            }
+            // ldmatrix.trans: lanes 0-7 keys 16kk..+7, 8-15 keys +8..+15 (dims 8jj..),
+            // lanes 16-31 the same keys at dims 8jj + 8
+            const int key = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+            const int dcol = (lane >> 4) * 8;
+#pragma unroll
+            for (int jj = 0; jj < NT; jj += 2) {
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_trans(ptx::smem_u32(&sm.v[stage][key][jj * 8 + dcol]), b0, b1, b2, b3);
+                mma_16816(o[jj], ah, b0, b1);
+                mma_16816(o[jj], al, b0, b1);
+                mma_16816(o[jj + 1], ah, b2, b3);
+                mma_16816(o[jj + 1], al, b2, b3);
+            }
+        }
+        __syncthreads();  // every warp is done with this stage before it is refilled
+    }
+#pragma unroll
+    for (int x = 1; x <= 2; x <<= 1) {
+        lA += __shfl_xor_sync(0xffffffffu, lA, x);
+        lB += __shfl_xor_sync(0xffffffffu, lB, x);
     }
 
-    const int64_t out_row = int64_t(m) * p.H * D;
     if (splits == 1) {
-        if (warp < nh) {
-            const float inv = __fdiv_rn(1.0f, run_l);
-            __nv_bfloat16* o = p.O + out_row + int64_t(h0 + warp) * D + lane * DL;
+        const float iA = __fdiv_rn(1.0f, lA), iB = __fdiv_rn(1.0f, lB);
 #pragma unroll
-            for (int d = 0; d < DL; d += 2)
-                *reinterpret_cast<__nv_bfloat162*>(o + d) =
-                    __floats2bfloat162_rn(__fmul_rn(acc[d], inv), __fmul_rn(acc[d + 1], inv));
+        for (int j = 0; j < NT; ++j) {
+            const int c = j * 8 + 2 * qc;
+            if (offA >= 0)
+                *reinterpret_cast<__nv_bfloat162*>(p.O + offA + c) =
+                    __floats2bfloat162_rn(__fmul_rn(o[j][0], iA), __fmul_rn(o[j][1], iA));
+            if (offB >= 0)
+                *reinterpret_cast<__nv_bfloat162*>(p.O + offB + c) =
+                    __floats2bfloat162_rn(__fmul_rn(o[j][2], iB), __fmul_rn(o[j][3], iB));
         }
         return;
     }
-    // split combine through distributed shared memory
-    if (warp < nh) {
-        if (lane == 0) {
-            sm.part_m[warp] = run_m;
-            sm.part_l[warp] = run_l;
-        }
+    // partials of this split into shared memory, then the cluster combines them
+    const int lrA = warp * 16 + quad, lrB = lrA + 8;
 #pragma unroll
-        for (int d = 0; d < DL; ++d) sm.part_o[warp][lane * DL + d] = acc[d];
+    for (int j = 0; j < NT; ++j) {
+        const int c = j * 8 + 2 * qc;
+        sm.part_o[lrA][c] = o[j][0];
+        sm.part_o[lrA][c + 1] = o[j][1];
+        sm.part_o[lrB][c] = o[j][2];
+        sm.part_o[lrB][c + 1] = o[j][3];
+    }
+    if (qc == 0) {
+        sm.part_m[lrA] = mA;
+        sm.part_l[lrA] = lA;
+        sm.part_m[lrB] = mB;
+        sm.part_l[lrB] = lB;
     }
     ptx::cluster_sync();
-    // CTA z combines the heads w with w % splits == z (warp w of this CTA does head w)
-    if (warp < nh && warp % splits == z) {
-        const uint32_t pm = ptx::smem_u32(&sm.part_m[warp]);
-        const uint32_t pl = ptx::smem_u32(&sm.part_l[warp]);
-        const uint32_t po = ptx::smem_u32(&sm.part_o[warp][lane * DL]);
-        // every split's partials are read before any is used (one remote round trip)
-        float qm[8], ql[8], qo[8][DL];
+    // CTA z combines rows [z * 64 / splits, (z + 1) * 64 / splits): one thread per 4 dims
+    const int rows_per = kAttnRows / splits;
+    for (int e = threadIdx.x; e < rows_per * (D / 4); e += kAttnThreads) {
+        const int lr = z * rows_per + e / (D / 4), c = (e % (D / 4)) * 4;
+        const int64_t off = q_row(row0 + lr);
+        if (off < 0) continue;
+        const uint32_t am = ptx::smem_u32(&sm.part_m[lr]), al_ = ptx::smem_u32(&sm.part_l[lr]);
+        const uint32_t ao = ptx::smem_u32(&sm.part_o[lr][c]);
+        float qm[8], ql[8];
+        float4 qo[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             if (q < splits) {
-                qm[q] = ptx::ld_dsmem_f32(ptx::map_dsmem(pm, q));
-                ql[q] = ptx::ld_dsmem_f32(ptx::map_dsmem(pl, q));
-#pragma unroll
-                for (int d = 0; d < DL; ++d) qo[q][d] = ptx::ld_dsmem_f32(ptx::map_dsmem(po + 4 * d, q));
+                qm[q] = ptx::ld_dsmem_f32(ptx::map_dsmem(am, q));
+                ql[q] = ptx::ld_dsmem_f32(ptx::map_dsmem(al_, q));
+                qo[q] = ptx::ld_dsmem_f32x4(ptx::map_dsmem(ao, q));
             }
         }
         float mx = -INFINITY;
 #pragma unroll
         for (int q = 0; q < 8; ++q)
             if (q < splits) mx = fmaxf(mx, qm[q]);
-        float L = 0.0f, O[DL];
-#pragma unroll
-        for (int d = 0; d < DL; ++d) O[d] = 0.0f;
+        float L = 0.0f;
+        float4 O = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             if (q < splits && qm[q] != -INFINITY) {  // a split without keys adds nothing
                 const float w = expf(qm[q] - mx);
                 L = fmaf(ql[q], w, L);
-#pragma unroll
-                for (int d = 0; d < DL; ++d) O[d] = fmaf(qo[q][d], w, O[d]);
+                O.x = fmaf(qo[q].x, w, O.x);
+                O.y = fmaf(qo[q].y, w, O.y);
+                O.z = fmaf(qo[q].z, w, O.z);
+                O.w = fmaf(qo[q].w, w, O.w);
             }
         }
         const float inv = __fdiv_rn(1.0f, L);
-        __nv_bfloat16* o = p.O + out_row + int64_t(h0 + warp) * D + lane * DL;
-#pragma unroll
-        for (int d = 0; d < DL; d += 2)
-            *reinterpret_cast<__nv_bfloat162*>(o + d) =
-                __floats2bfloat162_rn(__fmul_rn(O[d], inv), __fmul_rn(O[d + 1], inv));
+        const __nv_bfloat162 lo = __floats2bfloat162_rn(__fmul_rn(O.x, inv), __fmul_rn(O.y, inv));
+        const __nv_bfloat162 hi = __floats2bfloat162_rn(__fmul_rn(O.z, inv), __fmul_rn(O.w, inv));
+        uint2 u;
+        u.x = *reinterpret_cast<const uint32_t*>(&lo);
+        u.y = *reinterpret_cast<const uint32_t*>(&hi);
+        *reinterpret_cast<uint2*>(p.O + off + c) = u;
     }
     ptx::cluster_sync();  // remote shared memory must outlive its readers
 }
@@ -361,9 +448,10 @@ cudaError_t launch_attention_d(const AttnParams& p, int splits, cudaStream_t s) 
     }
     AttnParams pc = p;
     void* args[] = {&pc};
+    const int64_t row_blocks = (int64_t(p.M) * (p.H / p.Hk) + kAttnRows - 1) / kAttnRows;
     return launch_pdl(reinterpret_cast<const void*>(attention_kernel<D>),
-                      dim3(p.M, p.Hk * p.subgroups, splits), dim3(kAttnThreads), smem, s, args,
-                      unsigned(splits));
+                      dim3(unsigned(row_blocks), unsigned(p.Hk), unsigned(splits)), dim3(kAttnThreads),
+                      smem, s, args, unsigned(splits));
 }
 
 }  // namespace
@@ -413,10 +501,8 @@ cudaError_t launch_attention(const uint16_t* Q, const uint16_t* K0, const uint16
     p.M = int(M);
     p.H = int(H);
     p.Hk = int(Hk);
-    const int G = int(H / Hk);
-    p.subgroups = (G + kAttnWarps - 1) / kAttnWarps;
     p.scale = scale;
-    // key splits (one cluster): at least 64 keys each, at most 8 (the portable cluster size)
+    // key splits (one cluster): at least 128 keys each, at most 8 (the portable cluster size)
     const int64_t n = n0 + n1;
     int splits = 1;
     while (splits < 8 && n >= int64_t(splits) * 2 * kKeyTile) splits *= 2;
