@@ -25,6 +25,7 @@ from __future__ import annotations
 import argparse
 import concurrent.futures as cf
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -575,13 +576,284 @@ def measure_e2e(chains, args, dev, dist, tensor_bound):
                    "of the recorded chain, one D2H copy of all outputs; synchronise each step"}
 
 
+# ------------------------------------------------------------------ whole-layer loops
+
+LAYER_LOOPS = {"action_expert_layers": wl.action_expert_layers}
+
+
+class LayerLoopState:
+    """Device state of a LayerLoop: per layer its packed weights, norm gains and prefix
+    cache; one residual stream and one buffer per intermediate, reused by every layer."""
+
+    def __init__(self, L: "wl.LayerLoop", dev):
+        import torch
+        import paper_2607_02501_gb300 as emb
+        self.L, self.dev = L, dev
+        g = torch.Generator(device="cpu")
+        self.imgs, self.g1, self.g2, self.K0, self.V0 = [], [], [], [], []
+        for l in range(L.layers):
+            imgs = {}
+            for lin in L.linears(l):
+                W = wl.weight_torch(lin, device=dev)
+                imgs[lin.name.rsplit(".", 1)[1]] = emb.quantize(L.fmt, W)
+                del W
+            self.imgs.append(imgs)
+            g.manual_seed(L.seed0 + 16 * l + 8)
+            self.g1.append((1.0 + 0.1 * torch.randn(L.D, generator=g)).to(dev))
+            self.g2.append((1.0 + 0.1 * torch.randn(L.D, generator=g)).to(dev))
+            self.K0.append(torch.randn(L.prefix, L.Hk * L.d, generator=g).to(torch.bfloat16).to(dev))
+            self.V0.append(torch.randn(L.prefix, L.Hk * L.d, generator=g).to(torch.bfloat16).to(dev))
+        g.manual_seed(L.seed0 + 1)
+        self.R0 = (torch.randn(L.M, L.D, generator=g) * 2.0)
+        self.R = self.R0.to(dev)
+        bf = lambda *sh: torch.zeros(*sh, dtype=torch.bfloat16, device=dev)
+        M = L.M
+        self.h, self.h2 = bf(M, L.D), bf(M, L.D)
+        self.q, self.k, self.v = bf(M, L.H * L.d), bf(M, L.Hk * L.d), bf(M, L.Hk * L.d)
+        self.a, self.gg = bf(M, L.H * L.d), bf(M, L.F)
+        torch.cuda.synchronize()
+
+    def layer(self, l, s, parts=("norm", "linear", "rope", "attention")):
+        import paper_2607_02501_gb300 as emb
+        L, w, fmt = self.L, self.imgs[l], self.L.fmt
+        M, D, F = L.M, L.D, L.F
+        qd, kd = L.H * L.d, L.Hk * L.d
+        if "norm" in parts:
+            emb.emb_rmsnorm(self.R, self.g1[l], self.h, 1e-6, stream=s)
+        if "linear" in parts:
+            emb.emb_qlayer_seq_chained([(fmt, w["q"], qd, D, self.h, self.q, emb.EMB_EPI_BF16),
+                                (fmt, w["k"], kd, D, self.h, self.k, emb.EMB_EPI_BF16),
+                                (fmt, w["v"], kd, D, self.h, self.v, emb.EMB_EPI_BF16)], M, stream=s)
+        if "rope" in parts:
+            emb.emb_rope(self.q, L.H, L.d, L.prefix, 10000.0, stream=s)
+            emb.emb_rope(self.k, L.Hk, L.d, L.prefix, 10000.0, stream=s)
+        if "attention" in parts:
+            emb.emb_attention(self.q, self.K0[l], self.V0[l], self.k, self.v, self.a, L.H, L.Hk,
+                              L.d, 1.0 / math.sqrt(L.d), stream=s)
+        if "linear" in parts:
+            emb.emb_qlayer_seq_chained([(fmt, w["o"], D, qd, self.a, self.R, emb.EMB_EPI_ADD)], M, stream=s)
+        if "norm" in parts:
+            emb.emb_rmsnorm(self.R, self.g2[l], self.h2, 1e-6, stream=s)
+        if "linear" in parts:
+            emb.emb_qlayer_seq_chained([(fmt, w["gate_up"], 2 * F, D, self.h2, self.gg, emb.EMB_EPI_GEGLU)], M,
+                               stream=s)
+            emb.emb_qlayer_seq_chained([(fmt, w["down"], D, F, self.gg, self.R, emb.EMB_EPI_ADD)], M, stream=s)
+
+    def record(self, s, parts=("norm", "linear", "rope", "attention")):
+        """The loop (steps x layers) recorded as one chain on stream s."""
+        import paper_2607_02501_gb300 as emb
+        rec = emb.Recording(s)
+        with rec:
+            for _ in range(self.L.steps):
+                for l in range(self.L.layers):
+                    self.layer(l, s, parts)
+        return rec
+
+
+def layer_loop_oracle(L, budget_s: float):
+    """The oracle over one layer of the loop (its six matmuls from oracle-packed weights,
+    two norms, two rotaries, attention), repeated for about budget_s; flop/s."""
+    import numpy as np
+    import oracle
+    import torch
+    rng = np.random.default_rng(3)
+    imgs = []
+    for lin in L.linears(0):
+        W = wl.weight_torch(lin, device="cpu").numpy()
+        imgs.append((lin, oracle.quantize(L.fmt, W)))
+    bf = lambda *sh: oracle.bf16_round(rng.standard_normal(sh))
+    R = rng.standard_normal((L.M, L.D)).astype(np.float32)
+    gam = np.ones(L.D, dtype=np.float32)
+    K0, V0 = bf(L.prefix, L.Hk * L.d), bf(L.prefix, L.Hk * L.d)
+    to_bits = lambda x: torch.from_numpy(np.asarray(x, dtype=np.float32)).to(torch.bfloat16).view(
+        torch.int16).numpy().view(np.uint16)
+    t0 = time.perf_counter()
+    rounds = 0
+    while True:
+        h, _ = oracle.rmsnorm_reference(R, gam, 1e-6)
+        hb = to_bits(h)
+        outs = {}
+        for lin, img in imgs[:3]:
+            outs[lin.name.rsplit(".", 1)[1]] = oracle.qmatmul(L.fmt, img, hb, lin.N, lin.K)[0]
+        q, _ = oracle.rope_reference(oracle.bf16_round(outs["q"]), L.H, L.d, L.prefix, 10000.0)
+        k, _ = oracle.rope_reference(oracle.bf16_round(outs["k"]), L.Hk, L.d, L.prefix, 10000.0)
+        a, _ = oracle.attention_reference(q, K0, V0, k, oracle.bf16_round(outs["v"]), L.H, L.Hk, L.d,
+                                          1.0 / math.sqrt(L.d))
+        lin, img = imgs[3]
+        Ro = R + oracle.qmatmul(L.fmt, img, to_bits(a), lin.N, lin.K)[0]
+        h2, _ = oracle.rmsnorm_reference(Ro.astype(np.float32), gam, 1e-6)
+        lin, img = imgs[4]
+        gu = oracle.qmatmul(L.fmt, img, to_bits(h2), lin.N, lin.K)[0]
+        gg, _ = oracle.epilogue_reference(oracle.EPI_GEGLU, gu, np.zeros_like(gu))
+        lin, img = imgs[5]
+        oracle.qmatmul(L.fmt, img, to_bits(gg), lin.N, lin.K)
+        rounds += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            return L.layer_flops() * rounds / el, el, rounds
+
+
+def run_layer_loop(args):
+    import torch
+    import paper_2607_02501_gb300 as emb
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = init_dist(world, "nccl")
+    emb.lib()
+    L = LAYER_LOOPS[args.workload]()
+    st = LayerLoopState(L, dev)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        for l in range(L.layers):      # one eager pass (per-device setup happens here)
+            st.layer(l, s)
+        s.synchronize()
+        full = st.record(s)
+        # the same loop with only the linears, and with only the attention: the roofline's
+        # per-launch figures for the kernel families
+        lin_only = st.record(s, ("linear",))
+        attn_only = st.record(s, ("attention",))
+    torch.cuda.synchronize()
+    assert emb.emb_device_status() == emb.EMB_OK
+
+    def timed(rec, steps):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+        with torch.cuda.stream(s):
+            ev[0].record(s)
+            for i in range(steps):
+                rec.launch(s)
+                ev[i + 1].record(s)
+        torch.cuda.synchronize()
+        return ev[0].elapsed_time(ev[-1])
+
+    with torch.cuda.stream(s):
+        for _ in range(args.warmup):
+            full.launch(s)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
+    barrier(dist)
+    torch.cuda.synchronize()
+    total_ms = timed(full, args.steps)
+    barrier(dist)
+    clocks = sampler.stop()
+    assert emb.emb_device_status() == emb.EMB_OK
+    max_ms = max_over_ranks(total_ms, dist, dev)
+    value = world * L.flops() * args.steps / (max_ms / 1e3) / 1e12
+
+    # kernel families timed on their own (same launches, same buffers)
+    k_steps = max(3, min(args.steps, 20))
+    lin_ms = timed(lin_only, k_steps) / k_steps
+    attn_ms = timed(attn_only, k_steps) / k_steps
+    assert emb.emb_device_status() == emb.EMB_OK
+    peaks = load_peaks()
+    lin_launches = 4 * L.layers * L.steps
+    lin_bytes = sum(lin.N * lin.K // 32 * wl.BLOCK_BYTES[L.fmt] for lin in L.linears(0)) * L.layers * L.steps
+    if lin_ms >= attn_ms:
+        per_launch = lin_ms / lin_launches
+        achieved = lin_bytes / lin_launches / (per_launch / 1e3) / 1e9
+        kernel = "gemm_tc_kernel <Q8_0> (q/k/v, o, gate/up, down)"
+        nl = lin_launches
+    else:
+        qd, kd = L.H * L.d, L.Hk * L.d
+        ab = 2 * L.M * qd * 2 + 2 * 2 * (L.prefix + L.M) * kd
+        per_launch = attn_ms / (L.layers * L.steps)
+        achieved = ab / (per_launch / 1e3) / 1e9
+        kernel = "attention_kernel <128>"
+        nl = L.layers * L.steps
+    roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": kernel,
+            "peak_source": f"{peaks['source']} HBM copy bandwidth",
+            "launches_per_step": nl, "per_launch_us": per_launch * 1e3,
+            "family_ms_per_step": {"linears": lin_ms, "attention": attn_ms}}
+
+    # e2e: per closed-loop step the host supplies the chunk's starting residual stream and
+    # reads back the final one; the loop replays on the device in between
+    host_r = st.R0.pin_memory()
+    host_out = torch.empty_like(host_r).pin_memory()
+    e2e_steps = max(1, min(args.steps, 100))
+    with torch.cuda.stream(s):
+        for _ in range(2):
+            st.R.copy_(host_r, non_blocking=True)
+            full.launch(s)
+            host_out.copy_(st.R, non_blocking=True)
+        s.synchronize()
+        barrier(dist)
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            st.R.copy_(host_r, non_blocking=True)
+            full.launch(s)
+            host_out.copy_(st.R, non_blocking=True)
+            s.synchronize()
+        el = max_over_ranks(time.perf_counter() - t0, dist, dev)
+    e2e = {"value": world * L.flops() * e2e_steps / el / 1e12, "unit": "TFLOP/s",
+           "h2d_bytes_per_step": host_r.numel() * 4, "d2h_bytes_per_step": host_out.numel() * 4,
+           "steps": e2e_steps, "ms_per_step": el / e2e_steps * 1e3,
+           "how": "one pinned H2D copy of the starting residual, one replay of the recorded loop, "
+                  "one D2H copy of the final residual; synchronise each step"}
+    line = {"metric": "whole-layer loop TFLOP/s (linears + attention), M=50",
+            "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": max_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.workload, "formats": [wl.FMT_NAMES[L.fmt]], "M": L.M,
+                       "layers": L.layers, "denoise_steps": L.steps, "prefix_tokens": L.prefix,
+                       "heads": [L.H, L.Hk, L.d], "flops_per_step": L.flops(),
+                       "algorithmic_bytes_per_step": L.algorithmic_bytes(),
+                       "l2": "weights per step 274 MB > 126 MB L2",
+                       "parallelism": f"replica x{world}"},
+            "roofline": roof, "e2e": e2e, "clocks": clocks,
+            "gpu_launches": L.launches() * args.steps}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        fps, el_o, rounds = layer_loop_oracle(L, 8.0)
+        line["cpu_baseline"] = {"value": fps / 1e12, "unit": "TFLOP/s", "cores": oracle.host_threads(),
+                                "kind": "oracle",
+                                "sample": f"one layer of the loop (six matmuls, two norms, two "
+                                          f"rotaries, attention) x{rounds} over {el_o:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line))
+    full.close()
+    lin_only.close()
+    attn_only.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_layer_loop_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    L = LAYER_LOOPS[args.workload]()
+    per_step = min(2.0, 90.0 / max(1, args.steps + args.warmup))
+    layer_loop_oracle(L, per_step * args.warmup)
+    fps, el, rounds = layer_loop_oracle(L, per_step * args.steps)
+    value = fps / 1e12
+    sample = f"each step: the oracle over one layer of the loop, {rounds} layers in {el:.1f} s"
+    line = {"impl": "reference", "metric": "whole-layer loop TFLOP/s (linears + attention), M=50",
+            "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "M": L.M, "layers": L.layers},
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": oracle.host_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="gemma2b_decode")
+    ap.add_argument("--workload", choices=sorted(list(WORKLOADS) + list(LAYER_LOOPS)),
+                    default="gemma2b_decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first L layers (small cases for ncu captures; "
@@ -589,6 +861,10 @@ def main(argv=None):
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.workload in LAYER_LOOPS:
+        if args.layers:
+            ap.error("--layers applies to the linear-chain workloads")
+        return run_layer_loop_reference(args) if args.impl == "reference" else run_layer_loop(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)

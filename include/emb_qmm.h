@@ -180,6 +180,16 @@ EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, 
 EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M,
                           void* workspace, size_t ws_bytes, emb_stream_t stream);
 
+/* As emb_qlayer_seq, for a call inside a chain of this library's launches (a layer's
+ * linears between its norm, rotary and attention launches): the first launch of the call
+ * also overlaps its weight fetch with the end of the launch before it on `stream`, as
+ * every later launch of a call does. Precondition: the weights of the call are not
+ * written by the launch enqueued on `stream` just before the call (weights produced
+ * further back, e.g. by emb_quantize_* followed by any other launch or a synchronisation,
+ * are fine). Results are bitwise those of emb_qlayer_seq. Errors as emb_qlayer_seq. */
+EMB_API emb_status emb_qlayer_seq_chained(const emb_qlayer* layers, int n_layers, int64_t M,
+                                          emb_stream_t stream);
+
 /* ------------------------------------------------------------ recorded chains
  * Graph replay and buffer reuse (Section 3.2, design principle 2): the
  * launches that emb_qlayer_seq(layers, n_layers, M, workspace, ws_bytes, ...) enqueues

@@ -103,6 +103,8 @@ def lib():
     L.emb_status_string.restype = ctypes.c_char_p
     L.emb_build_info.argtypes = []
     L.emb_build_info.restype = ctypes.c_char_p
+    L.emb_qlayer_seq_chained.argtypes = [ctypes.POINTER(emb_qlayer), i32, i64, vp]
+    L.emb_qlayer_seq_chained.restype = i32
     L.emb_chain_record_begin.argtypes = [vp]
     L.emb_chain_record_begin.restype = i32
     L.emb_chain_record_end.argtypes = [vp, ctypes.POINTER(vp)]
@@ -197,6 +199,13 @@ def emb_qlayer_seq(layers, M: int, workspace=None, ws_bytes: int = 0, stream=Non
     arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
     _check(lib().emb_qlayer_seq(arr, len(arr), M, _ptr(workspace), ws_bytes, _stream(stream)),
            "emb_qlayer_seq")
+
+
+def emb_qlayer_seq_chained(layers, M: int, stream=None) -> None:
+    """emb_qlayer_seq whose first launch also overlaps the previous launch on the stream
+    (the call's weights must not be written by that launch)."""
+    arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
+    _check(lib().emb_qlayer_seq_chained(arr, len(arr), M, _stream(stream)), "emb_qlayer_seq_chained")
 
 
 def emb_chain_create(layers, M: int, workspace=None, ws_bytes: int = 0) -> int:

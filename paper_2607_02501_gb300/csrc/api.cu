@@ -251,12 +251,12 @@ static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
     return EMB_OK;
 }
 
-static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s) {
+static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s, bool first_pdl) {
     for (size_t i = 0; i < refs.size(); ++i) {
         // the first launch must not overlap whatever the caller enqueued before (it may
-        // have produced the weights); later ones overlap their weight fetch with the
-        // previous launch of this chain
-        const cudaError_t e = launch_group(refs[i], i > 0, s);
+        // have produced the weights) unless the caller says it did not; later ones overlap
+        // their weight fetch with the previous launch of this chain
+        const cudaError_t e = launch_group(refs[i], i > 0 || first_pdl, s);
         if (e != cudaSuccess) return EMB_ECUDA;
     }
     return EMB_OK;
@@ -269,7 +269,15 @@ emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, voi
     std::vector<GroupRef> refs;
     const emb_status st = prepare_seq(layers, n_layers, M, refs);
     if (st != EMB_OK) return st;
-    return enqueue_seq(refs, reinterpret_cast<cudaStream_t>(stream));
+    return enqueue_seq(refs, reinterpret_cast<cudaStream_t>(stream), false);
+}
+
+emb_status emb_qlayer_seq_chained(const emb_qlayer* layers, int n_layers, int64_t M,
+                                  emb_stream_t stream) {
+    std::vector<GroupRef> refs;
+    const emb_status st = prepare_seq(layers, n_layers, M, refs);
+    if (st != EMB_OK) return st;
+    return enqueue_seq(refs, reinterpret_cast<cudaStream_t>(stream), true);
 }
 
 }  // extern "C"
@@ -300,7 +308,7 @@ emb_status emb_chain_create(const emb_qlayer* layers, int n_layers, int64_t M, v
         cudaStreamDestroy(s);
         return EMB_ECUDA;
     }
-    st = enqueue_seq(refs, s);
+    st = enqueue_seq(refs, s, false);
     const cudaError_t ec = cudaStreamEndCapture(s, &graph);  // ends the capture in every case
     if (st == EMB_OK && ec != cudaSuccess) st = EMB_ECUDA;
     if (st == EMB_OK && cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) st = EMB_ECUDA;

@@ -127,20 +127,20 @@ def test_action_expert_layer_recorded(cuda_device):
     scale = 1.0 / math.sqrt(d)
     s = torch.cuda.Stream()
 
-    def part1(stream):
+    def part1(stream, seq=emb.emb_qlayer_seq):
         emb.emb_rmsnorm(dev["R"], dev["g1"], h, 1e-6, stream=stream)
-        emb.emb_qlayer_seq([(fmt, imgs["q"], H * d, D, h, q, emb.EMB_EPI_BF16),
+        seq([(fmt, imgs["q"], H * d, D, h, q, emb.EMB_EPI_BF16),
                             (fmt, imgs["k"], Hk * d, D, h, k, emb.EMB_EPI_BF16),
                             (fmt, imgs["v"], Hk * d, D, h, v, emb.EMB_EPI_BF16)], M, stream=stream)
         emb.emb_rope(q, H, d, P, 10000.0, stream=stream)
         emb.emb_rope(k, Hk, d, P, 10000.0, stream=stream)
         emb.emb_attention(q, dev["K0"], dev["V0"], k, v, a, H, Hk, d, scale, stream=stream)
-        emb.emb_qlayer_seq([(fmt, imgs["o"], D, H * d, a, dev["R"], emb.EMB_EPI_ADD)], M, stream=stream)
+        seq([(fmt, imgs["o"], D, H * d, a, dev["R"], emb.EMB_EPI_ADD)], M, stream=stream)
 
-    def part2(stream):
+    def part2(stream, seq=emb.emb_qlayer_seq):
         emb.emb_rmsnorm(dev["R"], dev["g2"], h2, 1e-6, stream=stream)
-        emb.emb_qlayer_seq([(fmt, imgs["gu"], 2 * F, D, h2, gg, emb.EMB_EPI_GEGLU)], M, stream=stream)
-        emb.emb_qlayer_seq([(fmt, imgs["d"], D, F, gg, dev["R"], emb.EMB_EPI_ADD)], M, stream=stream)
+        seq([(fmt, imgs["gu"], 2 * F, D, h2, gg, emb.EMB_EPI_GEGLU)], M, stream=stream)
+        seq([(fmt, imgs["d"], D, F, gg, dev["R"], emb.EMB_EPI_ADD)], M, stream=stream)
 
     # eager, with the residual kept between the halves, checked step by step against the
     # oracle, each step from the bits the GPU produced before it
@@ -188,8 +188,9 @@ def test_action_expert_layer_recorded(cuda_device):
     r_, b_ = oracle.epilogue_reference(oracle.EPI_ADD, Y, B, R1n)
     _check(dev["R"].cpu().numpy().astype(np.float64), r_, b_, "down + residual")
 
-    # the whole layer recorded as one chain: nothing runs while recording, and a replay
-    # gives the eager run's bits
+    # the whole layer recorded as one chain, its linears through emb_qlayer_seq_chained (the
+    # first launch of each call overlapping the layer step before it): nothing runs while
+    # recording, and a replay gives the eager run's bits
     eager = [t.clone() for t in (h, q, k, v, a, h2, gg, dev["R"])]
     dev["R"].copy_(torch.from_numpy(R0))
     for t in (h, q, k, v, a, h2, gg):
@@ -199,8 +200,8 @@ def test_action_expert_layer_recorded(cuda_device):
     with torch.cuda.stream(s):
         rec = emb.Recording(s)
         with rec:
-            part1(s)
-            part2(s)
+            part1(s, emb.emb_qlayer_seq_chained)
+            part2(s, emb.emb_qlayer_seq_chained)
     torch.cuda.synchronize()
     assert torch.isnan(h.float()).all() and torch.equal(dev["R"].cpu(), torch.from_numpy(R0))
     for _ in range(2):

@@ -216,3 +216,73 @@ def bf16_bits_np(x: np.ndarray) -> np.ndarray:
 def activation_bits_np(M: int, K: int, seed: int) -> np.ndarray:
     x = np.random.default_rng(seed).standard_normal((M, K)).astype(np.float32)
     return bf16_bits_np(x)
+
+
+@dataclasses.dataclass(frozen=True)
+class LayerLoop:
+    """Whole transformer layers run as a loop (the action expert's flow-matching steps):
+    per step, `layers` layers of RMSNorm -> q/k/v (bf16) -> rotary -> attention over the
+    layer's prefix key/value cache plus the chunk's own keys -> o (+ residual) -> RMSNorm ->
+    gate/up (interleaved rows, GeGLU, bf16) -> down (+ residual). Every step reuses the
+    layers' weights, caches and buffers."""
+    name: str
+    fmt: int
+    M: int          # chunk tokens
+    D: int          # width
+    H: int          # query heads
+    Hk: int         # key/value heads
+    d: int          # head dim
+    F: int          # ffn width (gate/up has 2F interleaved rows)
+    prefix: int     # prefix cache tokens (the chunk sits at positions prefix .. prefix + M - 1)
+    layers: int
+    steps: int
+    seed0: int
+
+    def linears(self, layer: int):
+        """The layer's matrices: q, k, v, o, gate_up (2F interleaved rows), down."""
+        s = self.seed0 + 16 * layer
+        a = f"{self.name}.L{layer}"
+        return [Linear(f"{a}.q", self.H * self.d, self.D, s + 0),
+                Linear(f"{a}.k", self.Hk * self.d, self.D, s + 1),
+                Linear(f"{a}.v", self.Hk * self.d, self.D, s + 2),
+                Linear(f"{a}.o", self.D, self.H * self.d, s + 3),
+                Linear(f"{a}.gate_up", 2 * self.F, self.D, s + 4),
+                Linear(f"{a}.down", self.D, self.F, s + 6)]
+
+    def layer_flops(self) -> int:
+        mm = sum(2 * self.M * lin.N * lin.K for lin in self.linears(0))
+        attn = 4 * self.M * self.H * (self.prefix + self.M) * self.d   # q.k and p.v
+        return mm + attn
+
+    def layer_bytes(self) -> int:
+        """Algorithmic bytes of one layer: weights once, every activation read and written
+        once, the prefix cache and the chunk's keys/values read once."""
+        M, D, F = self.M, self.D, self.F
+        qd, kd = self.H * self.d, self.Hk * self.d
+        w = sum(lin.N * lin.K // 32 * BLOCK_BYTES[self.fmt] for lin in self.linears(0))
+        norm = 2 * (4 * M * D + 4 * D + 2 * M * D)               # two norms: residual, gamma, out
+        qkv = 2 * M * D + 2 * M * (qd + 2 * kd)                  # read h, write q, k, v
+        rope = 2 * 2 * M * (qd + kd)                             # q, k read and written
+        attn = 2 * M * qd + 2 * 2 * (self.prefix + M) * kd + 2 * M * qd
+        o = 2 * M * qd + 8 * M * D                                # read a, residual add
+        gu = 2 * M * D + 2 * M * F                                # read h2, write GeGLU output
+        down = 2 * M * F + 8 * M * D
+        return w + norm + qkv + rope + attn + o + gu + down
+
+    def flops(self) -> int:
+        return self.layer_flops() * self.layers * self.steps
+
+    def algorithmic_bytes(self) -> int:
+        return self.layer_bytes() * self.layers * self.steps
+
+    def launches(self) -> int:
+        """Kernel launches of one loop: norm, q/k/v, rotary q, rotary k, attention, o, norm,
+        gate/up, down per layer."""
+        return 9 * self.layers * self.steps
+
+
+def action_expert_layers(steps: int = 10) -> LayerLoop:
+    """The action expert (width 1024, 8 query heads and 1 key/value head of 128, ffn 4096,
+    18 layers) over an 816-token prefix cache (3 x 256 image + 48 text tokens), M = 50,
+    Q8_0, 10 denoising steps."""
+    return LayerLoop("action_expert_layers", Q8_0, 50, 1024, 8, 1, 128, 4096, 816, 18, steps, 7000)
