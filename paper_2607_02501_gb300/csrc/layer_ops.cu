@@ -144,6 +144,8 @@ constexpr int kAttnWarps = 4;
 constexpr int kAttnThreads = 32 * kAttnWarps;
 constexpr int kAttnRows = 16 * kAttnWarps;
 constexpr int kKeyTile = 64;
+constexpr int kMaxSplits = 16;      // cluster size along the keys (16: non-portable, opted in)
+constexpr int kMinSplitKeys = 48;   // keys per split, at least
 
 template <int D>
 struct AttnSmem {
@@ -396,10 +398,10 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __grid_co
         if (off < 0) continue;
         const uint32_t am = ptx::smem_u32(&sm.part_m[lr]), al_ = ptx::smem_u32(&sm.part_l[lr]);
         const uint32_t ao = ptx::smem_u32(&sm.part_o[lr][c]);
-        float qm[8], ql[8];
-        float4 qo[8];
+        float qm[kMaxSplits], ql[kMaxSplits];
+        float4 qo[kMaxSplits];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
+        for (int q = 0; q < kMaxSplits; ++q) {
             if (q < splits) {
                 qm[q] = ptx::ld_dsmem_f32(ptx::map_dsmem(am, q));
                 ql[q] = ptx::ld_dsmem_f32(ptx::map_dsmem(al_, q));
@@ -408,12 +410,12 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __grid_co
         }
         float mx = -INFINITY;
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
+        for (int q = 0; q < kMaxSplits; ++q)
             if (q < splits) mx = fmaxf(mx, qm[q]);
         float L = 0.0f;
         float4 O = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
+        for (int q = 0; q < kMaxSplits; ++q) {
             if (q < splits && qm[q] != -INFINITY) {  // a split without keys adds nothing
                 const float w = expf(qm[q] - mx);
                 L = fmaf(ql[q], w, L);
@@ -444,6 +446,10 @@ cudaError_t launch_attention_d(const AttnParams& p, int splits, cudaStream_t s) 
     if (dev < 0 || dev >= 64 || !attr_done[dev]) {
         e = cudaFuncSetAttribute(attention_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         if (e != cudaSuccess) return e;
+        if (kMaxSplits > 8) {
+            e = cudaFuncSetAttribute(attention_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+            if (e != cudaSuccess) return e;
+        }
         if (dev >= 0 && dev < 64) attr_done[dev] = true;
     }
     AttnParams pc = p;
@@ -502,10 +508,10 @@ cudaError_t launch_attention(const uint16_t* Q, const uint16_t* K0, const uint16
     p.H = int(H);
     p.Hk = int(Hk);
     p.scale = scale;
-    // key splits (one cluster): at least 128 keys each, at most 8 (the portable cluster size)
+    // key splits (one cluster): at least kMinSplitKeys keys each, at most kMaxSplits
     const int64_t n = n0 + n1;
     int splits = 1;
-    while (splits < 8 && n >= int64_t(splits) * 2 * kKeyTile) splits *= 2;
+    while (splits < kMaxSplits && n >= int64_t(2 * splits) * kMinSplitKeys) splits *= 2;
     return D == 64 ? launch_attention_d<64>(p, splits, s) : launch_attention_d<128>(p, splits, s);
 }
 
