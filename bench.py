@@ -625,8 +625,7 @@ class LayerLoopState:
                                 (fmt, w["k"], kd, D, self.h, self.k, emb.EMB_EPI_BF16),
                                 (fmt, w["v"], kd, D, self.h, self.v, emb.EMB_EPI_BF16)], M, stream=s)
         if "rope" in parts:
-            emb.emb_rope(self.q, L.H, L.d, L.prefix, 10000.0, stream=s)
-            emb.emb_rope(self.k, L.Hk, L.d, L.prefix, 10000.0, stream=s)
+            emb.emb_rope_qk(self.q, L.H, self.k, L.Hk, L.d, L.prefix, 10000.0, stream=s)
         if "attention" in parts:
             emb.emb_attention(self.q, self.K0[l], self.V0[l], self.k, self.v, self.a, L.H, L.Hk,
                               L.d, 1.0 / math.sqrt(L.d), stream=s)

@@ -258,6 +258,13 @@ EMB_API emb_status emb_rmsnorm(const float* x, const float* gamma, uint16_t* y, 
 EMB_API emb_status emb_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim,
                             int64_t pos0, float base, emb_stream_t stream);
 
+/* emb_rope of q [M][n_q_heads][head_dim] and k [M][n_k_heads][head_dim] at the same
+ * positions in one launch (results bitwise those of two emb_rope calls). k may be NULL
+ * when n_k_heads == 0; q and k may not overlap. Errors as emb_rope. */
+EMB_API emb_status emb_rope_qk(uint16_t* q, int64_t n_q_heads, uint16_t* k, int64_t n_k_heads,
+                               int64_t M, int64_t head_dim, int64_t pos0, float base,
+                               emb_stream_t stream);
+
 /* Scaled dot-product attention (Vaswani et al., 2017) of M query tokens over n0 + n1 keys:
  * the prefix cache (K0, V0: [n0][n_kv_heads][head_dim]) followed by the chunk's own keys
  * (K1, V1: [n1][n_kv_heads][head_dim]), all visible to every query (no mask). Query head h

@@ -114,6 +114,8 @@ def lib():
     L.emb_rmsnorm.restype = i32
     L.emb_rope.argtypes = [vp, i64, i64, i64, i64, f32, vp]
     L.emb_rope.restype = i32
+    L.emb_rope_qk.argtypes = [vp, i64, vp, i64, i64, i64, i64, f32, vp]
+    L.emb_rope_qk.restype = i32
     L.emb_attention.argtypes = [vp, vp, vp, i64, vp, vp, i64, vp, i64, i64, i64, i64, f32, vp]
     L.emb_attention.restype = i32
     _lib = L
@@ -308,6 +310,13 @@ def emb_rope(x, n_heads: int, head_dim: int, pos0: int, base: float = 10000.0, s
     """In place on bf16 x [M][n_heads * head_dim]; token m at position pos0 + m."""
     _check(lib().emb_rope(_ptr(x), x.shape[0], n_heads, head_dim, pos0, base, _stream(stream)),
            "emb_rope")
+
+
+def emb_rope_qk(q, n_q_heads: int, k, n_k_heads: int, head_dim: int, pos0: int,
+                base: float = 10000.0, stream=None) -> None:
+    """emb_rope of q and k (same positions) in one launch."""
+    _check(lib().emb_rope_qk(_ptr(q), n_q_heads, _ptr(k), n_k_heads, q.shape[0], head_dim, pos0, base,
+                             _stream(stream)), "emb_rope_qk")
 
 
 def emb_attention(Q, K0, V0, K1, V1, O, n_heads: int, n_kv_heads: int, head_dim: int,

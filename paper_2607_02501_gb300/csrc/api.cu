@@ -370,15 +370,25 @@ emb_status emb_rmsnorm(const float* x, const float* gamma, uint16_t* y, int64_t 
     return from_cuda(launch_rmsnorm(x, gamma, y, M, D, eps, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+emb_status emb_rope_qk(uint16_t* q, int64_t n_q_heads, uint16_t* k, int64_t n_k_heads, int64_t M,
+                       int64_t head_dim, int64_t pos0, float base, emb_stream_t stream) {
+    if (!q || M < 1 || n_q_heads < 1 || n_k_heads < 0 || (n_k_heads > 0 && !k) || head_dim < 2 ||
+        head_dim % 2 != 0 || head_dim > 512 || pos0 < 0 || pos0 + M > (int64_t(1) << 24) ||
+        M * (n_q_heads + n_k_heads) * head_dim >= (int64_t(1) << 46) || !(base > 0.0f) ||
+        !std::isfinite(base))
+        return EMB_EINVAL;
+    if (!aligned(q, 16) || (n_k_heads > 0 && !aligned(k, 16))) return EMB_EALIGN;
+    if (n_k_heads > 0 &&
+        overlap(Range{uintptr_t(q), uintptr_t(q) + uintptr_t(M * n_q_heads * head_dim * 2)},
+                Range{uintptr_t(k), uintptr_t(k) + uintptr_t(M * n_k_heads * head_dim * 2)}))
+        return EMB_EINVAL;
+    return from_cuda(launch_rope(q, n_q_heads, n_k_heads > 0 ? k : nullptr, n_k_heads, M, head_dim, pos0,
+                                 double(base), reinterpret_cast<cudaStream_t>(stream)));
+}
+
 emb_status emb_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim, int64_t pos0,
                     float base, emb_stream_t stream) {
-    if (!x || M < 1 || n_heads < 1 || head_dim < 2 || head_dim % 2 != 0 || head_dim > 512 ||
-        pos0 < 0 || pos0 + M > (int64_t(1) << 24) || M * n_heads * head_dim >= (int64_t(1) << 46) ||
-        !(base > 0.0f) || !std::isfinite(base))
-        return EMB_EINVAL;
-    if (!aligned(x, 16)) return EMB_EALIGN;
-    return from_cuda(launch_rope(x, M, n_heads, head_dim, pos0, double(base),
-                                 reinterpret_cast<cudaStream_t>(stream)));
+    return emb_rope_qk(x, n_heads, nullptr, 0, M, head_dim, pos0, base, stream);
 }
 
 emb_status emb_attention(const uint16_t* Q, const uint16_t* K0, const uint16_t* V0, int64_t n0,

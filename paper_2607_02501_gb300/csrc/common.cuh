@@ -142,8 +142,8 @@ bool gemm_tc_supported(const GroupRef& g);
 // chunk's own keys. Arguments are validated by the caller (api.cu).
 cudaError_t launch_rmsnorm(const float* x, const float* gamma, uint16_t* y, int64_t M, int64_t D,
                            float eps, cudaStream_t s);
-cudaError_t launch_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim, int64_t pos0,
-                        double base, cudaStream_t s);
+cudaError_t launch_rope(uint16_t* x, int64_t n_heads, uint16_t* x2, int64_t n_heads2, int64_t M,
+                        int64_t head_dim, int64_t pos0, double base, cudaStream_t s);
 cudaError_t launch_attention(const uint16_t* Q, const uint16_t* K0, const uint16_t* V0, int64_t n0,
                              const uint16_t* K1, const uint16_t* V1, int64_t n1, uint16_t* O,
                              int64_t M, int64_t H, int64_t Hk, int64_t D, float scale, cudaStream_t s);

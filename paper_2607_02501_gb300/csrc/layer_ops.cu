@@ -99,9 +99,10 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __re
 constexpr int kRopeMaxPairs = 256;
 
 struct RopeParams {
-    __nv_bfloat16* x;
-    int64_t pairs, pos0;
-    int n_heads, head_dim;
+    __nv_bfloat16* x;   // [M][n_heads][head_dim]
+    __nv_bfloat16* x2;  // [M][n_heads2][head_dim] at the same positions, or nothing (n_heads2 = 0)
+    int64_t pairs1, pairs, pos0;
+    int n_heads, n_heads2, head_dim;
     float inv_hi[kRopeMaxPairs], inv_lo[kRopeMaxPairs];
 };
 
@@ -109,9 +110,12 @@ __global__ void __launch_bounds__(256) rope_kernel(const __grid_constant__ RopeP
     ptx::griddep_launch_dependents();
     ptx::griddep_wait();  // x was written by the previous launch
     const int half = p.head_dim / 2;
-    const int64_t per_token = int64_t(p.n_heads) * half;
-    for (int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; t < p.pairs;
-         t += int64_t(gridDim.x) * blockDim.x) {
+    for (int64_t t0 = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; t0 < p.pairs;
+         t0 += int64_t(gridDim.x) * blockDim.x) {
+        const bool second = t0 >= p.pairs1;  // the pairs of x come first, then those of x2
+        const int64_t t = second ? t0 - p.pairs1 : t0;
+        const int heads = second ? p.n_heads2 : p.n_heads;
+        const int64_t per_token = int64_t(heads) * half;
         const int64_t m = t / per_token;
         const int r = int(t - m * per_token);
         const int h = r / half, i = r - h * half;
@@ -121,7 +125,7 @@ __global__ void __launch_bounds__(256) rope_kernel(const __grid_constant__ RopeP
         float sA, cA;
         sincosf(A, &sA, &cA);
         const float c = fmaf(-a, sA, cA), s = fmaf(a, cA, sA);
-        __nv_bfloat16* xp = p.x + m * (int64_t(p.n_heads) * p.head_dim) + int64_t(h) * p.head_dim + i;
+        __nv_bfloat16* xp = (second ? p.x2 : p.x) + m * (int64_t(heads) * p.head_dim) + int64_t(h) * p.head_dim + i;
         const float xa = __bfloat162float(xp[0]), xb = __bfloat162float(xp[half]);
         xp[0] = __float2bfloat16_rn(__fsub_rn(__fmul_rn(xa, c), __fmul_rn(xb, s)));
         xp[half] = __float2bfloat16_rn(__fadd_rn(__fmul_rn(xb, c), __fmul_rn(xa, s)));
@@ -473,13 +477,16 @@ cudaError_t launch_rmsnorm(const float* x, const float* gamma, uint16_t* y, int6
                       dim3(kNormThreads), 0, s, args);
 }
 
-cudaError_t launch_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim, int64_t pos0,
-                        double base, cudaStream_t s) {
+cudaError_t launch_rope(uint16_t* x, int64_t n_heads, uint16_t* x2, int64_t n_heads2, int64_t M,
+                        int64_t head_dim, int64_t pos0, double base, cudaStream_t s) {
     RopeParams p;
     p.x = reinterpret_cast<__nv_bfloat16*>(x);
-    p.pairs = M * n_heads * (head_dim / 2);
+    p.x2 = reinterpret_cast<__nv_bfloat16*>(x2);
+    p.pairs1 = M * n_heads * (head_dim / 2);
+    p.pairs = p.pairs1 + M * n_heads2 * (head_dim / 2);
     p.pos0 = pos0;
     p.n_heads = int(n_heads);
+    p.n_heads2 = int(n_heads2);
     p.head_dim = int(head_dim);
     for (int i = 0; i < kRopeMaxPairs; ++i) {
         const double v = i < head_dim / 2 ? std::pow(base, -2.0 * double(i) / double(head_dim)) : 0.0;

@@ -17,7 +17,7 @@ def L():
 
 def test_every_declared_symbol_is_exported(L):
     names = emb.declared_symbols()
-    assert len(names) == 22
+    assert len(names) == 23
     for n in names:
         assert hasattr(L, n), n
 
@@ -233,3 +233,10 @@ def test_rope_validation(L, args, expect):
 def test_attention_validation(L, args, expect):
     assert L.emb_attention(*args, None) == expect
 
+
+
+def test_rope_qk_validation(L):
+    assert L.emb_rope_qk(A, 8, None, 1, 50, 128, 816, 1e4, None) == emb.EMB_EINVAL      # k missing
+    assert L.emb_rope_qk(A, 8, A + 4096, 1, 50, 128, 816, 1e4, None) == emb.EMB_EINVAL  # k inside q
+    assert L.emb_rope_qk(A, 8, B + 2, 1, 50, 128, 816, 1e4, None) == emb.EMB_EALIGN     # k misaligned
+    assert L.emb_rope_qk(A, 8, B, -1, 50, 128, 816, 1e4, None) == emb.EMB_EINVAL        # negative heads

@@ -59,6 +59,23 @@ def test_rope_parity(cuda_device, M, H, d, pos0, base):
     _check(_vals(x), ref, bound, f"rope M={M} H={H} d={d} pos0={pos0}")
 
 
+@pytest.mark.parametrize("M,H,Hk,d", [(50, 8, 1, 128), (7, 3, 5, 64), (1, 1, 1, 2)])
+def test_rope_qk_is_two_ropes_in_one_launch(cuda_device, M, H, Hk, d):
+    rng = np.random.default_rng(M + H + Hk + d)
+    qb = oracle.bf16_round(rng.standard_normal((M, H * d)))
+    kb = oracle.bf16_round(rng.standard_normal((M, Hk * d)))
+    q1, k1, q2, k2 = _bf16_dev(qb), _bf16_dev(kb), _bf16_dev(qb), _bf16_dev(kb)
+    emb.emb_rope_qk(q1, H, k1, Hk, d, 816, 10000.0)
+    emb.emb_rope(q2, H, d, 816, 10000.0)
+    emb.emb_rope(k2, Hk, d, 816, 10000.0)
+    torch.cuda.synchronize()
+    assert torch.equal(q1.view(torch.int16), q2.view(torch.int16))
+    assert torch.equal(k1.view(torch.int16), k2.view(torch.int16))
+    for t, xb, heads in ((q1, qb, H), (k1, kb, Hk)):
+        ref, bound = oracle.rope_reference(xb, heads, d, 816, 10000.0)
+        _check(_vals(t), ref, bound, f"rope_qk heads={heads}")
+
+
 # (M, H, Hk, d, n0, n1): the action expert over the 816-token prefix; grouped heads with
 # two kv heads and no cache; 16 heads of one kv head (two CTAs of 8 heads); one kv head per
 # query head; a single key; many keys at one query (eight key splits); a ragged last tile
@@ -127,13 +144,16 @@ def test_action_expert_layer_recorded(cuda_device):
     scale = 1.0 / math.sqrt(d)
     s = torch.cuda.Stream()
 
-    def part1(stream, seq=emb.emb_qlayer_seq):
+    def part1(stream, seq=emb.emb_qlayer_seq, one_rope=False):
         emb.emb_rmsnorm(dev["R"], dev["g1"], h, 1e-6, stream=stream)
         seq([(fmt, imgs["q"], H * d, D, h, q, emb.EMB_EPI_BF16),
                             (fmt, imgs["k"], Hk * d, D, h, k, emb.EMB_EPI_BF16),
                             (fmt, imgs["v"], Hk * d, D, h, v, emb.EMB_EPI_BF16)], M, stream=stream)
-        emb.emb_rope(q, H, d, P, 10000.0, stream=stream)
-        emb.emb_rope(k, Hk, d, P, 10000.0, stream=stream)
+        if one_rope:
+            emb.emb_rope_qk(q, H, k, Hk, d, P, 10000.0, stream=stream)
+        else:
+            emb.emb_rope(q, H, d, P, 10000.0, stream=stream)
+            emb.emb_rope(k, Hk, d, P, 10000.0, stream=stream)
         emb.emb_attention(q, dev["K0"], dev["V0"], k, v, a, H, Hk, d, scale, stream=stream)
         seq([(fmt, imgs["o"], D, H * d, a, dev["R"], emb.EMB_EPI_ADD)], M, stream=stream)
 
@@ -200,7 +220,7 @@ def test_action_expert_layer_recorded(cuda_device):
     with torch.cuda.stream(s):
         rec = emb.Recording(s)
         with rec:
-            part1(s, emb.emb_qlayer_seq_chained)
+            part1(s, emb.emb_qlayer_seq_chained, one_rope=True)
             part2(s, emb.emb_qlayer_seq_chained)
     torch.cuda.synchronize()
     assert torch.isnan(h.float()).all() and torch.equal(dev["R"].cpu(), torch.from_numpy(R0))

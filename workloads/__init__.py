@@ -276,9 +276,9 @@ class LayerLoop:
         return self.layer_bytes() * self.layers * self.steps
 
     def launches(self) -> int:
-        """Kernel launches of one loop: norm, q/k/v, rotary q, rotary k, attention, o, norm,
+        """Kernel launches of one loop: norm, q/k/v, rotary of q and k, attention, o, norm,
         gate/up, down per layer."""
-        return 9 * self.layers * self.steps
+        return 8 * self.layers * self.steps
 
 
 def action_expert_layers(steps: int = 10) -> LayerLoop:
