@@ -10,6 +10,7 @@
 // only after griddepcontrol.wait, so it chains behind the layer launches of emb_qlayer_seq.
 #include <algorithm>
 #include <cmath>
+#include <mutex>
 
 #include "ptx.cuh"
 
@@ -443,10 +444,13 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __grid_co
 template <int D>
 cudaError_t launch_attention_d(const AttnParams& p, int splits, cudaStream_t s) {
     const size_t smem = sizeof(AttnSmem<D>);
+    // the opt-in shared-memory size and cluster size are per-device function attributes
+    static std::mutex mu;
     static bool attr_done[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
     if (dev < 0 || dev >= 64 || !attr_done[dev]) {
         e = cudaFuncSetAttribute(attention_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         if (e != cudaSuccess) return e;
