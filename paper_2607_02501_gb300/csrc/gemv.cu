@@ -165,7 +165,11 @@ __device__ __forceinline__ float dot_unit(const uint4 c, const uint2 h, const fl
     else return dot_q6_unit(c, h, x);
 }
 
-template <int FMT, int R, int NT, int MT>
+// PF > 1 (M = 1 only, U <= PF * NT): every unit of the thread is loaded into registers
+// before griddepcontrol.wait, so a layer with long rows has all of its weight bytes in
+// flight while the previous launch drains; the products are summed in the same order as
+// with PF = 1 (bitwise the same results).
+template <int FMT, int R, int NT, int MT, int PF>
 __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvParams p) {
     constexpr int UW = (FMT == EMB_Q8_0) ? 16 : 32;  // weights per 16-byte unit
     constexpr int NWARP = NT / 32;
@@ -205,16 +209,45 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
         }
     };
 
-    int u = t;
-    if (u < U) load_unit(u, c, h, d);
-    // weights do not depend on earlier launches; X and Y may
-    griddep_wait();
-
     float acc[R][MT];
 #pragma unroll
     for (int r = 0; r < R; ++r)
 #pragma unroll
         for (int j = 0; j < MT; ++j) acc[r][j] = 0.0f;
+
+    if constexpr (PF > 1) {
+        static_assert(MT == 1, "whole-row prefetch is for one token");
+        uint4 cp[PF][R];
+        uint2 hp[PF][R];
+        float dp[PF][R];
+#pragma unroll
+        for (int k = 0; k < PF; ++k)
+            if (t + k * NT < U) load_unit(t + k * NT, cp[k], hp[k], dp[k]);
+        // weights do not depend on earlier launches; X and Y may
+        griddep_wait();
+#pragma unroll
+        for (int k = 0; k < PF; ++k) {
+            const int uk = t + k * NT;
+            if (uk >= U) break;
+            float x[UW];
+            const uint4* xp = reinterpret_cast<const uint4*>(p.X + int64_t(m0) * p.K + int64_t(uk) * UW);
+#pragma unroll
+            for (int v = 0; v < UW / 8; ++v) {
+                const uint4 hx = __ldg(xp + v);
+                x[8 * v + 0] = lo_bf16(hx.x); x[8 * v + 1] = hi_bf16(hx.x);
+                x[8 * v + 2] = lo_bf16(hx.y); x[8 * v + 3] = hi_bf16(hx.y);
+                x[8 * v + 4] = lo_bf16(hx.z); x[8 * v + 5] = hi_bf16(hx.z);
+                x[8 * v + 6] = lo_bf16(hx.w); x[8 * v + 7] = hi_bf16(hx.w);
+            }
+#pragma unroll
+            for (int r = 0; r < R; ++r) acc[r][0] = fmaf(dp[k][r], dot_unit<FMT>(cp[k][r], hp[k][r], x), acc[r][0]);
+        }
+    }
+
+    int u = (PF > 1) ? U : t;
+    if (u < U) load_unit(u, c, h, d);
+    // weights do not depend on earlier launches; X and Y may
+    if constexpr (PF == 1) griddep_wait();
 
     for (; u < U; u += NT) {
         uint4 cn[R];
@@ -283,7 +316,7 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
     }
 }
 
-template <int FMT, int R, int NT, int MT>
+template <int FMT, int R, int NT, int MT, int PF = 1>
 cudaError_t launch_one(const GemvParams& p, int grid_x, int grid_y, bool pdl, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid_x, grid_y, 1);
@@ -295,11 +328,18 @@ cudaError_t launch_one(const GemvParams& p, int grid_x, int grid_y, bool pdl, cu
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, gemv_kernel<FMT, R, NT, MT>, p);
+    return cudaLaunchKernelEx(&cfg, gemv_kernel<FMT, R, NT, MT, PF>, p);
 }
 
 template <int FMT, int R, int NT>
 cudaError_t dispatch_mt(const GemvParams& p, int grid_x, int M, bool pdl, cudaStream_t s) {
+    // Q8_0 rows longer than one pass of the CTA's threads (at most four) are loaded whole
+    // before the wait (measured on GB300, Gemma-2B decode chain at M = 1, whose down
+    // projection 2048 x 16384 takes this path: Q8_0 3899 -> 3987 GB/s). Not for Q4_0:
+    // its variant needs ~100 registers, halves the resident CTAs and lost (2265 -> 2068).
+    if constexpr (FMT == EMB_Q8_0 && R <= 2) {
+        if (M == 1 && p.U > NT && p.U <= 4 * NT) return launch_one<FMT, R, NT, 1, 4>(p, grid_x, 1, pdl, s);
+    }
     if (M == 1) return launch_one<FMT, R, NT, 1>(p, grid_x, 1, pdl, s);
     if (M == 2) return launch_one<FMT, R, NT, 2>(p, grid_x, 1, pdl, s);
     return launch_one<FMT, R, NT, 4>(p, grid_x, (M + 3) / 4, pdl, s);

@@ -13,9 +13,12 @@ pytestmark = pytest.mark.gpu
 
 FMTS = [emb.EMB_Q8_0, emb.EMB_Q4_0]
 
+# (1, 130, 16384), (1, 300, 11008) and (1, 1300, 7168) take the Q8_0 register kernel that
+# loads a thread's whole row share before the wait (1 to 4 passes, ragged last pass);
+# (1, 64, 40960) has rows longer than four passes and streams them one unit ahead.
 GEMV_SHAPES = [(1, 1, 32), (1, 8, 64), (1, 136, 96), (1, 256, 2048), (1, 2048, 2048),
-               (1, 130, 16384), (1, 300, 11008), (1, 4096, 1152), (2, 200, 4608),
-               (3, 129, 1024), (4, 1000, 2080)]
+               (1, 130, 16384), (1, 300, 11008), (1, 1300, 7168), (1, 64, 40960),
+               (1, 4096, 1152), (2, 200, 4608), (3, 129, 1024), (4, 1000, 2080)]
 
 GEMM_SHAPES = [(5, 128, 1024), (7, 136, 96), (16, 8, 32), (49, 256, 2048), (50, 1024, 1024),
                (51, 264, 1152), (64, 384, 256), (127, 128, 1088), (129, 640, 2048),
@@ -37,9 +40,9 @@ def test_gemm_parity(cuda_device, fmt, M, N, K):
     check_close(Y, Yref, B, f"gemm fmt={fmt} M={M} N={N} K={K}")
 
 
-@pytest.mark.parametrize("M", [1, 3, 50, 280])
-def test_deterministic(cuda_device, M):
-    N, K = 384, 2048
+@pytest.mark.parametrize("M,N,K", [(1, 384, 2048), (3, 384, 2048), (50, 384, 2048),
+                                   (280, 384, 2048), (1, 1300, 7168)])
+def test_deterministic(cuda_device, M, N, K):
     W = torch.from_numpy(weight_np(N, K, 3)).cuda()
     X = to_dev_bf16(activation_bits_np(M, K, 4))
     for fmt in FMTS:
