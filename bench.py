@@ -163,7 +163,8 @@ def summarize_clocks(rows):
 
 WORKLOADS = {
     "gemma2b_decode": lambda: [wl.gemma2b_decode(wl.Q8_0), wl.gemma2b_decode(wl.Q4_0)],
-    "single_linear": lambda: [wl.single_linear()],
+    # the 2048 x 2048 Q8_0 linear, 100 calls per step on distinct weight copies
+    "single_linear": lambda: [wl.single_linear_copies()],
     "action_expert": lambda: [wl.action_expert_denoise()],
     # the flow-matching loop recorded as one chain (10 steps x 18 layers, fused epilogues)
     "action_expert_fused": lambda: [wl.action_expert_fused()],
@@ -327,13 +328,16 @@ def cpu_baseline(workloads, budget_s=8.0, layers=2):
     import oracle
     threads = oracle.host_threads()
     total_bytes, total_t = 0.0, 0.0
+    n_lin = []
     for w in workloads:
         work = oracle_sample_images(w, min(layers, w.layers))
+        n_lin.append(len(work))
         bps, el, rounds = time_oracle(work, w.fmt, w.M, budget_s / len(workloads))
         total_bytes += bps * el
         total_t += el
-    sample = (f"first {layers} of {workloads[0].layers} layers "
-              f"({7 * layers} linears) per format, repeated over ~{budget_s:.0f} s; "
+    used = min(layers, workloads[0].layers)
+    sample = (f"first {used} of {workloads[0].layers} layers "
+              f"({'/'.join(map(str, n_lin))} linears) per format, repeated over ~{budget_s:.0f} s; "
               f"fp64 oracle matmul from oracle-packed weights, {threads} host threads")
     return {"value": total_bytes / total_t / 1e9, "unit": "GB/s", "cores": threads,
             "kind": "oracle", "sample": sample}
@@ -493,6 +497,7 @@ def run_ours(args):
     roof["per_launch_us"] = per_launch_ms * 1e3
 
     e2e = measure_e2e(chains, args, dev, dist, tensor_bound)
+    isolated = isolated_launch_us(chains[0]["specs"], ws[0].M) if args.workload == "single_linear" else None
 
     gpu_launches = sum(cc["launches"] * cc["w"].repeats for cc in chains) * args.steps
     line = {"metric": metric_name(ws), "value": value, "unit": unit, "n_gpus": world,
@@ -507,6 +512,8 @@ def run_ours(args):
                     (cc["flops"] if tensor_bound else cc["bytes"]) * cc["w"].repeats * args.steps
                     / (chain_ms[k] / 1e3) / (1e12 if tensor_bound else 1e9)}
                 for k, cc in enumerate(chains)}}
+    if isolated is not None:
+        line["isolated_launch_us"] = isolated
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         torch.cuda.synchronize()
         line["cpu_baseline"] = cpu_baseline(ws)
@@ -515,6 +522,25 @@ def run_ours(args):
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def isolated_launch_us(specs, M, n=50):
+    """One linear at a time on an idle GPU: device time between CUDA events around one
+    emb_qlayer_seq call (one launch), each call on the next weight copy; median and min."""
+    import torch
+    import paper_2607_02501_gb300 as emb
+    times = []
+    for i in range(n):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record()
+        emb.emb_qlayer_seq([specs[i % len(specs)]], M)
+        b.record()
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b) * 1e3)
+    times.sort()
+    return {"median": times[len(times) // 2], "min": times[0], "calls": n,
+            "how": "CUDA events around one emb_qlayer_seq call on an idle GPU, rotating weight copies"}
 
 
 def kernel_traffic(workload, w):

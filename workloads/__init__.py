@@ -114,6 +114,14 @@ def single_linear() -> Workload:
                     [[Linear("w", 2048, 2048, 1)]])
 
 
+def single_linear_copies(copies: int = 100) -> Workload:
+    """The single 2048x2048 Q8_0 linear at M=1 as a chain of `copies` calls, each on its own
+    copy of the weights and activation (seeds 1 .. copies), so that together the copies
+    (100 x 4.46 MB) exceed three times the 126 MB L2 and HBM serves every call."""
+    return Workload(f"single_q8_0_2048x2048_m1_x{copies}", Q8_0, 1, 1,
+                    tuple((Linear(f"w{i}", 2048, 2048, 1 + i),) for i in range(copies)))
+
+
 def gemma2b_decode(fmt: int) -> Workload:
     """Gemma-style 2B decoder linears, 18 layers, hidden 2048, kv 256, ffn 16384, M=1."""
     return Workload(f"gemma2b_decode_{FMT_NAMES[fmt].lower()}_m1", fmt, 1, 18,
