@@ -402,6 +402,32 @@ def metric_name(ws) -> str:
     return "qmatmul µs & HBM GB/s (M=1) / TFLOP/s (M≥50), as fraction of roofline"
 
 
+L2_BYTES = 126e6   # GB300 L2
+
+
+def distinct_weight_bytes(ws) -> int:
+    """Packed bytes of the distinct weight matrices a step reads (a loop that reuses a
+    layer's weights, as the denoising steps do, counts them once)."""
+    seen, total = set(), 0
+    for w in ws:
+        for lin in w.linears():
+            key = (w.fmt, lin.name, lin.N, lin.K, lin.seed)
+            if key not in seen:
+                seen.add(key)
+                total += lin.N * lin.K // 32 * wl.BLOCK_BYTES[w.fmt]
+    return total
+
+
+def l2_policy(distinct: int) -> str:
+    """How the timed steps keep weights from being served by L2 between reads."""
+    if distinct > 3 * L2_BYTES:
+        return "inputs larger than L2 (distinct weights per step >> 126 MB L2)"
+    if distinct > 2 * L2_BYTES:
+        return ("weights rotate through L2 (distinct weights per step > 2 x 126 MB L2, "
+                "read in the same order every pass)")
+    return "weights partly L2-resident (distinct weights per step < 2 x 126 MB L2)"
+
+
 def config_of(ws, args):
     w0 = ws[0]
     return {"workload": args.workload,
@@ -409,8 +435,8 @@ def config_of(ws, args):
             "M": w0.M, "layers": w0.layers, "linears_per_format": len(w0.linears()),
             "repeats": w0.repeats,
             "weight_bytes_per_step": sum(w.weight_bytes() * w.repeats for w in ws),
-            "l2": "inputs larger than L2 (weights per step >> 126 MB L2)"
-            if sum(w.weight_bytes() for w in ws) > 400e6 else "weights rotate through L2",
+            "distinct_weight_bytes": distinct_weight_bytes(ws),
+            "l2": l2_policy(distinct_weight_bytes(ws)),
             "parallelism": f"replica x{int(os.environ.get('WORLD_SIZE', '1'))}"}
 
 
@@ -464,6 +490,7 @@ def run_ours(args):
     total_ms = ev[0][0].elapsed_time(ev[-1][-1])
     chain_ms = [sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(args.steps))
                 for j in range(len(chains))]
+    per_step = step_stats([ev[i][0].elapsed_time(ev[i][-1]) for i in range(args.steps)])
     assert emb.emb_device_status() == emb.EMB_OK
     max_ms = max_over_ranks(total_ms, dist, dev)
 
@@ -512,6 +539,7 @@ def run_ours(args):
                     (cc["flops"] if tensor_bound else cc["bytes"]) * cc["w"].repeats * args.steps
                     / (chain_ms[k] / 1e3) / (1e12 if tensor_bound else 1e9)}
                 for k, cc in enumerate(chains)}}
+    line["step_ms"] = per_step
     if isolated is not None:
         line["isolated_launch_us"] = isolated
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -522,6 +550,15 @@ def run_ours(args):
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def step_stats(ms):
+    """Median, minimum and maximum of the per-step device times (CUDA events at each
+    step's start and end on this rank)."""
+    v = sorted(float(x) for x in ms)
+    n = len(v)
+    med = v[n // 2] if n % 2 else 0.5 * (v[n // 2 - 1] + v[n // 2])
+    return {"median": med, "min": v[0], "max": v[-1], "steps": n}
 
 
 def isolated_launch_us(specs, M, n=50):
