@@ -307,16 +307,16 @@ def oracle_sample_images(w: wl.Workload, layers: int):
     return [(lin, img, xs[lin.name]) for lin, img in imgs]
 
 
-def time_oracle(work, fmt, M, budget_s: float, min_rounds: int = 1):
+def time_oracle(work, fmt, M, budget_s: float, min_rounds: int = 1, nthreads: int = 0):
     """Run the oracle matmul over `work` (list of (lin, img, X)) repeatedly until
-    budget_s has passed; returns (bytes/s, elapsed, rounds)."""
+    budget_s has passed; returns (bytes/s, elapsed, rounds). nthreads 0 = every host core."""
     import oracle
     nbytes = 0
     t0 = time.perf_counter()
     rounds = 0
     while True:
         for lin, img, X in work:
-            oracle.qmatmul(fmt, img, X, lin.N, lin.K)
+            oracle.qmatmul(fmt, img, X, lin.N, lin.K, nthreads)
             nbytes += lin.N * lin.K // 32 * wl.BLOCK_BYTES[fmt] + M * lin.K * 2 + M * lin.N * 4
         rounds += 1
         el = time.perf_counter() - t0
@@ -328,6 +328,7 @@ def cpu_baseline(workloads, budget_s=8.0, layers=2):
     import oracle
     threads = oracle.host_threads()
     total_bytes, total_t = 0.0, 0.0
+    one_bytes, one_t = 0.0, 0.0
     n_lin = []
     for w in workloads:
         work = oracle_sample_images(w, min(layers, w.layers))
@@ -335,12 +336,18 @@ def cpu_baseline(workloads, budget_s=8.0, layers=2):
         bps, el, rounds = time_oracle(work, w.fmt, w.M, budget_s / len(workloads))
         total_bytes += bps * el
         total_t += el
+        # the same sample on one host thread (a shorter budget: one linear at least)
+        bps1, el1, _ = time_oracle(work[:1], w.fmt, w.M, budget_s / 4 / len(workloads), nthreads=1)
+        one_bytes += bps1 * el1
+        one_t += el1
     used = min(layers, workloads[0].layers)
     sample = (f"first {used} of {workloads[0].layers} layers "
               f"({'/'.join(map(str, n_lin))} linears) per format, repeated over ~{budget_s:.0f} s; "
               f"fp64 oracle matmul from oracle-packed weights, {threads} host threads")
     return {"value": total_bytes / total_t / 1e9, "unit": "GB/s", "cores": threads,
-            "kind": "oracle", "sample": sample}
+            "kind": "oracle", "sample": sample,
+            "value_1core": one_bytes / one_t / 1e9,
+            "sample_1core": "the first linear of the same sample, repeated on one host thread"}
 
 
 # ------------------------------------------------------------------ arms
