@@ -29,8 +29,11 @@
  *     stream) without any host synchronisation, except emb_device_status.
  *   - Argument errors are reported BEFORE anything is enqueued. Launch errors
  *     return EMB_ECUDA. Device-side failures (a bounded wait that expired) are
- *     recorded in a device status word read by emb_device_status.
+ *     recorded in a device status word read by emb_device_status. After
+ *     EMB_ETIMEOUT the outputs of the calls enqueued since the last status read
+ *     are undefined, residual-add (EMB_EPI_ADD) buffers included.
  *   - Outputs are fully overwritten. Inputs and outputs must not overlap.
+ * Each entry point below names the paper passage it serves.
  */
 #ifndef EMB_QMM_H
 #define EMB_QMM_H
@@ -79,6 +82,7 @@ typedef enum {
 } emb_status;
 
 /* ---------------------------------------------------------------- packed weights
+ * Section 4, Table 3 (the 8-, 6- and 4-bit configurations whose weights these are).
  * Packed image of one [N][K] matrix (one caller allocation of
  * emb_qweight_bytes(fmt, N, K) bytes, 256-byte aligned, written only by
  * emb_quantize_*; callers may copy, save and reload it as plain bytes):
@@ -98,30 +102,44 @@ typedef enum {
  * Returns the byte size, or 0 when fmt is unknown, N < 1, K < 32 or K % 32 != 0. */
 EMB_API size_t emb_qweight_bytes(emb_qfmt fmt, int64_t N, int64_t K);
 
-/* Quantise fp32 W [N][K] (device, 16-byte aligned) into W_blocks (device,
+/* Section 4, Table 3 (8-bit column): the offline packing of one weight matrix.
+ * Quantise fp32 W [N][K] (device, 16-byte aligned) into W_blocks (device,
  * 256-byte aligned, emb_qweight_bytes(EMB_Q8_0, N, K) bytes). Offline step of
  * the path (packing weights once per model). NaN/Inf weights, and weights so
  * large that max|w|/127 overflows fp16, are outside the contract. */
 EMB_API emb_status emb_quantize_q8_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream);
 
-/* As emb_quantize_q8_0 for EMB_Q4_0 (m/-8 must not overflow fp16). */
+/* Section 4, Table 3 (4-bit column).
+ * As emb_quantize_q8_0 for EMB_Q4_0 (m/-8 must not overflow fp16). */
 EMB_API emb_status emb_quantize_q4_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream);
 
-/* As emb_quantize_q8_0 for EMB_Q6_0, the 6-bit configuration (Table 3, 6-bit column;
- * the paper gives no format, EMB_Q6_0 above is this library's definition). */
+/* Section 4, Table 3 (6-bit column; the paper gives no format, EMB_Q6_0 above is this
+ * library's definition). As emb_quantize_q8_0 for EMB_Q6_0. */
 EMB_API emb_status emb_quantize_q6_0(const float* W, int64_t N, int64_t K, void* W_blocks,
                              emb_stream_t stream);
 
 /* ---------------------------------------------------------------------- matmul
+ * Section 3.1, challenge 2 (batch-1, latency-first control steps: M = 1 decode, M = 50
+ * action chunks, M = 250..820 prefix prefill) on the Table 3 weight formats.
  * Y [M][N] fp32 = X [M][K] bf16  x  w'^T, w' the dequantised weights of W_blocks.
  * X, Y: device, 16-byte aligned; W_blocks as produced by emb_quantize_*.
- * Small M (action-token decode) runs a weight-streaming GEMV that dequantises in
- * registers; larger M (action-chunk denoising, prefix prefill) runs a tcgen05
+ * Small M (M <= 4, action-token decode) runs a weight-streaming GEMV that dequantises
+ * in registers; larger M (action-chunk denoising, prefix prefill) runs a tcgen05
  * tensor-core GEMM that dequantises shared-memory tiles to bf16.
- * Accuracy: |Y - Y_exact| <= 1e-3 * sum_k |w'[n][k] x[m][k]| + 1e-6 per element,
- * where Y_exact uses the same dequantised weights and the same bf16 X.
+ * Accuracy, per element, with Y_exact from the same dequantised weights w' and the
+ * same bf16 X, and S = sum_k |w'[n][k] x[m][k]|:
+ *   - M <= 4, or K < 1024:  |Y - Y_exact| <= 1e-3 * S + 1e-6 for every input (the GEMV's
+ *     products are exact; below K = 1024 the GEMM's operand is bf16(w') plus the bf16 of
+ *     its rounding remainder, relative error <= 2^-16);
+ *   - M > 4 and K >= 1024:  the GEMM's operand is bf16(w'), relative error <= 2^-8 per
+ *     weight (bf16's unit roundoff), so |Y - Y_exact| <= (2^-8 + 2^-12) * S + 1e-6 always
+ *     (operand rounding plus fp32 accumulation), and the 1e-3 * S + 1e-6 bound holds when
+ *     S is spread over many terms (every workload shape: observed error / S below 2e-4)
+ *     but can fail when a handful of terms dominate S. A layer whose epilogue
+ *     carries EMB_PRECISE_OPERAND (emb_qlayer_seq) gets the two-operand form at every K
+ *     and the 1e-3 * S + 1e-6 bound for every input, at about twice the tensor work.
  * Results are bitwise reproducible from call to call for a given shape. */
 EMB_API emb_status emb_qmatmul(emb_qfmt fmt, const void* W_blocks, const uint16_t* X, float* Y,
                        int64_t M, int64_t N, int64_t K, emb_stream_t stream);
@@ -146,9 +164,14 @@ typedef enum {
     EMB_EPI_SWIGLU = 4
 } emb_epilogue;
 
+/* Flag OR-ed into emb_qlayer.epilogue: run this layer's tensor-core GEMM (M > 4) with the
+ * two-operand weights bf16(w') + bf16(w' - bf16(w')) at every K, so that emb_qmatmul's
+ * 1e-3 * S + 1e-6 accuracy holds for every input (see emb_qmatmul). No effect at M <= 4. */
+#define EMB_PRECISE_OPERAND 0x100
+
 typedef struct {
     int32_t fmt;            /* emb_qfmt */
-    int32_t epilogue;       /* emb_epilogue */
+    int32_t epilogue;       /* emb_epilogue, optionally | EMB_PRECISE_OPERAND */
     const void* W_blocks;   /* packed image of W [N][K] */
     int64_t N;
     int64_t K;
@@ -158,8 +181,12 @@ typedef struct {
 
 #define EMB_MAX_LAYERS 4096
 
-/* Bytes of device workspace emb_qlayer_seq needs for these layers at this M
- * (0 is a valid answer). Returns (size_t)-1 for invalid arguments. */
+/* Section 3.2, principle 2 (buffer reuse: the caller owns every buffer of a chain,
+ * the library allocates nothing).
+ * Bytes of device workspace emb_qlayer_seq needs for these layers at this M. This build's
+ * kernels need none: the answer is 0 for every valid chain (so EMB_ENOSPC does not occur
+ * and the workspace arguments of emb_qlayer_seq / emb_chain_create are reserved).
+ * Returns (size_t)-1 for invalid arguments. */
 EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M);
 
 /* Run n_layers linears in order on `stream`, all with M tokens (the paper's
@@ -173,14 +200,14 @@ EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, 
  * the next projection), and layers may add into the same residual buffer in
  * turn. A layer's W_blocks may not overlap the Y of the same or an earlier
  * layer, and its X may not overlap its own Y (EMB_EINVAL); an unknown epilogue,
- * or a gated one with odd N, is EMB_EINVAL. The call enqueues kernels only (plus
- * memsets of the workspace), so it may be captured into a CUDA graph and
- * replayed. workspace: device, 256-byte aligned, >= emb_qlayer_seq_workspace()
- * bytes (may be NULL when that is 0). */
+ * or a gated one with odd N, is EMB_EINVAL. The call enqueues kernels only, so it may
+ * be captured into a CUDA graph and replayed. workspace / ws_bytes: reserved; this
+ * build reads neither (emb_qlayer_seq_workspace() is 0), NULL / 0 are fine. */
 EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M,
                           void* workspace, size_t ws_bytes, emb_stream_t stream);
 
-/* As emb_qlayer_seq, for a call inside a chain of this library's launches (a layer's
+/* Section 3.2, principle 2 (operator fusion across a layer's launches).
+ * As emb_qlayer_seq, for a call inside a chain of this library's launches (a layer's
  * linears between its norm, rotary and attention launches): the first launch of the call
  * also overlaps its weight fetch with the end of the launch before it on `stream`, as
  * every later launch of a call does. Precondition: the weights of the call are not
@@ -197,7 +224,8 @@ EMB_API emb_status emb_qlayer_seq_chained(const emb_qlayer* layers, int n_layers
  * step costs one host call instead of one per launch group. */
 typedef struct emb_chain_st* emb_chain_t;
 
-/* Record the chain. Arguments, validation and error codes are those of emb_qlayer_seq
+/* Section 3.2, principle 2 (graph replay, buffer reuse).
+ * Record the chain. Arguments, validation and error codes are those of emb_qlayer_seq
  * (nothing is launched: the launches are captured on a private stream of the current
  * device). The recording holds the layers' pointers: every replay reads the X buffers
  * and fully overwrites the Y buffers given here, so callers refill the X buffers between
@@ -209,15 +237,17 @@ typedef struct emb_chain_st* emb_chain_t;
 EMB_API emb_status emb_chain_create(const emb_qlayer* layers, int n_layers, int64_t M,
                             void* workspace, size_t ws_bytes, emb_chain_t* chain);
 
-/* Enqueue one replay of the recorded chain on `stream` (a stream of the device it was
+/* Section 3.2, principle 2 (graph replay: one host call per closed-loop step).
+ * Enqueue one replay of the recorded chain on `stream` (a stream of the device it was
  * recorded on). EMB_EINVAL for a NULL handle, EMB_ECUDA if the launch fails. */
 EMB_API emb_status emb_chain_launch(emb_chain_t chain, emb_stream_t stream);
 
-/* Free the recording (NULL is a no-op). Replays already enqueued still complete. */
+/* Section 3.2, principle 2 (graph replay). Free the recording (NULL is a no-op).
+ * Replays already enqueued still complete. */
 EMB_API emb_status emb_chain_destroy(emb_chain_t chain);
 
-/* Record any sequence of this library's calls as one chain (graph replay of a whole layer
- * or loop, Section 3.2 principle 2). After emb_chain_record_begin(stream), every library
+/* Section 3.2, principle 2: record any sequence of this library's calls as one chain
+ * (graph replay of a whole layer or loop). After emb_chain_record_begin(stream), every library
  * call made by this thread on `stream` is recorded instead of run (CUDA stream capture in
  * thread-local mode) until emb_chain_record_end(stream, &chain) returns the recording,
  * which emb_chain_launch replays and emb_chain_destroy frees. The recording holds every
@@ -228,6 +258,7 @@ EMB_API emb_status emb_chain_destroy(emb_chain_t chain);
  * Errors: EMB_EINVAL (NULL stream or chain pointer), EMB_ECUDA (capture could not begin or
  * end, or instantiation failed; *chain is then NULL). */
 EMB_API emb_status emb_chain_record_begin(emb_stream_t stream);
+/* Section 3.2, principle 2 (graph replay): end the recording begun on `stream`. */
 EMB_API emb_status emb_chain_record_end(emb_stream_t stream, emb_chain_t* chain);
 
 /* ---------------------------------------------------------------- layer steps
@@ -237,7 +268,8 @@ EMB_API emb_status emb_chain_record_end(emb_stream_t stream, emb_chain_t* chain)
  * All are enqueued on `stream` with programmatic dependent launch, like emb_qlayer_seq,
  * allocate nothing, and are deterministic. bf16 buffers hold bit patterns (uint16_t). */
 
-/* RMSNorm (Zhang and Sennrich, 2019) of every token of the fp32 residual stream:
+/* Section 3.2 (the shared backbone layer around the linears).
+ * RMSNorm (Zhang and Sennrich, 2019) of every token of the fp32 residual stream:
  * y[m][i] = bf16(x[m][i] / sqrt(mean_i x[m][i]^2 + eps) * gamma[i]), the mean and square
  * root in fp32 (correctly rounded square root and reciprocal), one bf16 rounding.
  * x: device fp32 [M][D]; gamma: device fp32 [D]; y: device bf16 [M][D]; 16-byte aligned.
@@ -246,7 +278,8 @@ EMB_API emb_status emb_chain_record_end(emb_stream_t stream, emb_chain_t* chain)
 EMB_API emb_status emb_rmsnorm(const float* x, const float* gamma, uint16_t* y, int64_t M,
                                int64_t D, float eps, emb_stream_t stream);
 
-/* Rotary position embedding (Su et al., 2021), rotate-half pairing, in place on bf16
+/* Section 3.2 (the shared backbone layer around the linears).
+ * Rotary position embedding (Su et al., 2021), rotate-half pairing, in place on bf16
  * x [M][n_heads][head_dim]: token m sits at position pos0 + m; in every head, element i
  * and element i + head_dim/2 (i < head_dim/2) are rotated by the angle
  * (pos0 + m) * base^(-2i/head_dim): (a, b) -> (a cos - b sin, b cos + a sin). The
@@ -258,14 +291,17 @@ EMB_API emb_status emb_rmsnorm(const float* x, const float* gamma, uint16_t* y, 
 EMB_API emb_status emb_rope(uint16_t* x, int64_t M, int64_t n_heads, int64_t head_dim,
                             int64_t pos0, float base, emb_stream_t stream);
 
-/* emb_rope of q [M][n_q_heads][head_dim] and k [M][n_k_heads][head_dim] at the same
+/* Section 3.2 (the shared backbone layer), principle 2 (fusion: one launch for q and k).
+ * emb_rope of q [M][n_q_heads][head_dim] and k [M][n_k_heads][head_dim] at the same
  * positions in one launch (results bitwise those of two emb_rope calls). k may be NULL
  * when n_k_heads == 0; q and k may not overlap. Errors as emb_rope. */
 EMB_API emb_status emb_rope_qk(uint16_t* q, int64_t n_q_heads, uint16_t* k, int64_t n_k_heads,
                                int64_t M, int64_t head_dim, int64_t pos0, float base,
                                emb_stream_t stream);
 
-/* Scaled dot-product attention (Vaswani et al., 2017) of M query tokens over n0 + n1 keys:
+/* Section 3.1 (the action chunk attends to the prefix cache: "prefix once, head many")
+ * and Section 3.2 (the shared backbone layer).
+ * Scaled dot-product attention (Vaswani et al., 2017) of M query tokens over n0 + n1 keys:
  * the prefix cache (K0, V0: [n0][n_kv_heads][head_dim]) followed by the chunk's own keys
  * (K1, V1: [n1][n_kv_heads][head_dim]), all visible to every query (no mask). Query head h
  * (Q: [M][n_heads][head_dim]) reads key/value head h / (n_heads / n_kv_heads);
@@ -279,28 +315,36 @@ EMB_API emb_status emb_attention(const uint16_t* Q, const uint16_t* K0, const ui
                                  int64_t head_dim, float scale, emb_stream_t stream);
 
 /* ---------------------------------------------------------------- test support
+ * Section 4, Table 3 (the weights of the 8-, 6- and 4-bit configurations, dequantised).
  * Dequantise W_blocks to fp32 [N][K] (w' exactly: the products are exact in fp32). */
 EMB_API emb_status emb_dequantize_f32(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
                               float* out, emb_stream_t stream);
 
-/* Dequantise to bf16 bit patterns [N][K]: one round-to-nearest-even of the exact fp32
+/* Section 4, Table 3. Dequantise to bf16 bit patterns [N][K]: one round-to-nearest-even
+ * of the exact fp32
  * w' -- the operand values the tensor-core GEMM feeds to its MMAs. */
 EMB_API emb_status emb_dequantize_bf16(emb_qfmt fmt, const void* W_blocks, int64_t N, int64_t K,
                                uint16_t* out, emb_stream_t stream);
 
-/* Synchronise `stream`, then return and clear the device status word: EMB_OK, or
- * EMB_ETIMEOUT if a kernel's bounded wait expired since the last call. */
+/* Section 3.2 (the deployment boundary reports device-side failures to the host).
+ * Read and clear the device status word in one atomic exchange enqueued on `stream`,
+ * then synchronise `stream` (only that stream): EMB_OK, or EMB_ETIMEOUT if a kernel's
+ * bounded wait expired since the last call. A timeout recorded by work on another stream
+ * that has not finished yet is reported by a later call. */
 EMB_API emb_status emb_device_status(emb_stream_t stream);
 
-/* Launch one block that waits on a shared-memory barrier that nothing completes,
+/* Section 3.2 (deployment boundary; test support for the failure path above).
+ * Launch one block that waits on a shared-memory barrier that nothing completes,
  * giving up after timeout_ns nanoseconds (1e3 .. 1e9): exercises the bounded-wait
  * error path; emb_device_status then returns EMB_ETIMEOUT. */
 EMB_API emb_status emb_selftest_wait_timeout(int64_t timeout_ns, emb_stream_t stream);
 
-/* Human-readable name of a status code (static string). */
+/* Section 3.2 (deployment boundary). Human-readable name of a status code (static
+ * string). */
 EMB_API const char* emb_status_string(emb_status status);
 
-/* Static string describing the build (target architecture, kernel variants). */
+/* Section 3.2 (backend abstraction: which backend this is). Static string describing
+ * the build (target architecture, kernel variants). */
 EMB_API const char* emb_build_info(void);
 
 #ifdef __cplusplus

@@ -33,6 +33,7 @@ EMB_ECUDA = 4
 EMB_ETIMEOUT = 5
 EMB_EUNSUPPORTED = 6
 EMB_MAX_LAYERS = 4096
+EMB_PRECISE_OPERAND = 0x100   # flag OR-ed into a layer's epilogue (two-operand tensor-core weights)
 
 # layer epilogues (emb_epilogue)
 EMB_EPI_F32 = 0

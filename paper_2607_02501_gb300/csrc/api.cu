@@ -17,6 +17,7 @@ namespace emb {
 namespace {
 
 __device__ int g_status_word;  // OR of kStatus* flags; read and cleared by emb_device_status
+__device__ int g_status_read;  // where emb_device_status's exchange leaves the value it read
 
 // Token counts up to this run the GEMV; above it, the tensor-core GEMM.
 constexpr int64_t kGemvMaxM = 4;
@@ -30,6 +31,20 @@ int* status_ptr() {
     if (!ptrs[dev]) {
         void* p = nullptr;
         if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+        ptrs[dev] = static_cast<int*>(p);
+    }
+    return ptrs[dev];
+}
+
+int* status_read_ptr() {
+    static std::mutex mu;
+    static int* ptrs[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!ptrs[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_read) != cudaSuccess) return nullptr;
         ptrs[dev] = static_cast<int*>(p);
     }
     return ptrs[dev];
@@ -52,10 +67,14 @@ bool valid_shape(int64_t M, int64_t N, int64_t K) {
 
 emb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? EMB_OK : EMB_ECUDA; }
 
-bool valid_epi(int epi) { return epi >= EMB_EPI_F32 && epi <= EMB_EPI_SWIGLU; }
+// An emb_qlayer.epilogue value: an emb_epilogue kind, optionally | EMB_PRECISE_OPERAND.
+int epi_kind(int epi) { return epi & ~EMB_PRECISE_OPERAND; }
+bool epi_precise(int epi) { return (epi & EMB_PRECISE_OPERAND) != 0; }
+bool valid_epi(int epi) { return epi_kind(epi) >= EMB_EPI_F32 && epi_kind(epi) <= EMB_EPI_SWIGLU; }
 
 // Bytes a layer's epilogue writes (and, for EMB_EPI_ADD, reads) at Y.
 int64_t y_bytes(int epi, int64_t M, int64_t N) {
+    epi = epi_kind(epi);
     if (epi == EMB_EPI_F32 || epi == EMB_EPI_ADD) return M * N * 4;
     if (epi == EMB_EPI_BF16) return M * N * 2;
     return M * (N / 2) * 2;  // gated: one bf16 per gate/up row pair
@@ -65,7 +84,7 @@ int64_t y_bytes(int epi, int64_t M, int64_t N) {
 emb_status check_layer(int fmt, int epi, const void* W, const uint16_t* X, const void* Y, int64_t M,
                        int64_t N, int64_t K) {
     if (!valid_fmt(fmt) || !valid_epi(epi) || !valid_shape(M, N, K)) return EMB_EINVAL;
-    if (epi >= EMB_EPI_GEGLU && N % 2 != 0) return EMB_EINVAL;
+    if (epi_kind(epi) >= EMB_EPI_GEGLU && N % 2 != 0) return EMB_EINVAL;
     if (!W || !X || !Y) return EMB_EINVAL;
     if (!aligned(W, 256) || !aligned(X, 16) || !aligned(Y, 16)) return EMB_EALIGN;
     const Layout L = layout_of(fmt, N, K);
@@ -89,6 +108,10 @@ cudaError_t launch_group(const GroupRef& g, bool pdl, cudaStream_t s) {
     if (g.M <= kGemvMaxM) return launch_gemv(g, pdl, st, s);
     return launch_gemm_tc(g, pdl, st, s);
 }
+
+// Read and clear the status word in one atomic step, on the caller's stream: a flag that a
+// kernel ORs in concurrently is either returned now or kept for the next read.
+__global__ void status_exchange_kernel(int* status, int* out) { *out = atomicExch(status, 0); }
 
 // ------------------------------------------------------------ self-test kernel
 __global__ void selftest_wait_kernel(uint64_t timeout_ns, int* status) {
@@ -218,11 +241,6 @@ static emb_status check_seq(const emb_qlayer* layers, int n_layers, int64_t M) {
     return EMB_OK;
 }
 
-size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M) {
-    if (check_seq(layers, n_layers, M) != EMB_OK) return size_t(-1);
-    return 0;
-}
-
 // Validation of one chain and its launch groups (nothing enqueued).
 static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
                               std::vector<GroupRef>& refs) {
@@ -235,7 +253,8 @@ static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
         const emb_qlayer& L0 = layers[gr.first];
         GroupRef g = {};
         g.fmt = L0.fmt;
-        g.epi = L0.epilogue;
+        g.epi = epi_kind(L0.epilogue);
+        g.precise = epi_precise(L0.epilogue);
         g.n_mats = gr.second - gr.first;
         for (int k = 0; k < g.n_mats; ++k) {
             const emb_qlayer& L = layers[gr.first + k];
@@ -251,6 +270,11 @@ static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
     return EMB_OK;
 }
 
+size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M) {
+    if (check_seq(layers, n_layers, M) != EMB_OK) return size_t(-1);
+    return 0;
+}
+
 static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s, bool first_pdl) {
     for (size_t i = 0; i < refs.size(); ++i) {
         // the first launch must not overlap whatever the caller enqueued before (it may
@@ -264,7 +288,7 @@ static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s,
 
 emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
                           size_t ws_bytes, emb_stream_t stream) {
-    (void)workspace;
+    (void)workspace;  // reserved: this build's kernels need no workspace
     (void)ws_bytes;
     std::vector<GroupRef> refs;
     const emb_status st = prepare_seq(layers, n_layers, M, refs);
@@ -291,7 +315,7 @@ extern "C" {
 
 emb_status emb_chain_create(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
                             size_t ws_bytes, emb_chain_t* chain) {
-    (void)workspace;
+    (void)workspace;  // reserved, as for emb_qlayer_seq
     (void)ws_bytes;
     if (!chain) return EMB_EINVAL;
     *chain = nullptr;
@@ -432,13 +456,17 @@ emb_status emb_dequantize_bf16(emb_qfmt fmt, const void* W_blocks, int64_t N, in
 
 emb_status emb_device_status(emb_stream_t stream) {
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (cudaStreamSynchronize(s) != cudaSuccess) return EMB_ECUDA;
     int* st = status_ptr();
-    if (!st) return EMB_ECUDA;
+    int* slot = status_read_ptr();
+    if (!st || !slot) return EMB_ECUDA;
+    // one read slot per device: concurrent callers take turns
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    status_exchange_kernel<<<1, 1, 0, s>>>(st, slot);
+    if (cudaGetLastError() != cudaSuccess) return EMB_ECUDA;
     int host = 0;
-    if (cudaMemcpy(&host, st, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return EMB_ECUDA;
-    if (cudaMemset(st, 0, sizeof(int)) != cudaSuccess) return EMB_ECUDA;
-    if (cudaDeviceSynchronize() != cudaSuccess) return EMB_ECUDA;
+    if (cudaMemcpyAsync(&host, slot, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess) return EMB_ECUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return EMB_ECUDA;
     return (host & kStatusTimeout) ? EMB_ETIMEOUT : EMB_OK;
 }
 

@@ -119,7 +119,8 @@ struct MatRef {
 
 struct GroupRef {
     int fmt;
-    int epi;                // emb_epilogue of every member
+    int epi;                // emb_epilogue kind of every member (flags stripped)
+    bool precise;           // EMB_PRECISE_OPERAND: two-operand weights in the tensor-core GEMM
     int n_mats;
     MatRef mats[kMaxGroup];
     const __nv_bfloat16* X;

@@ -31,10 +31,10 @@
 // lets every copy and MMA it issued land, frees TMEM and returns.
 //
 // Precision: each operand value is bf16(w') -- one rounding of the exact fp32 w' -- so
-// the products are exact and accumulate in fp32. For K < 1024 the SPLIT variant also
-// stages lo = bf16(w' - bf16(w')) and issues a second MMA per step, which brings the
-// operand error from 2^-9 to 2^-17 relative (the 1e-3 * sum|w x| bound then holds for
-// every input, not only statistically).
+// the products are exact and accumulate in fp32. For K < 1024, and for layers flagged
+// EMB_PRECISE_OPERAND, the SPLIT variant also stages lo = bf16(w' - bf16(w')) and issues
+// a second MMA per step, which brings the operand error from 2^-8 to 2^-16 relative (the
+// 1e-3 * sum|w x| bound then holds for every input, not only statistically).
 #include <cuda.h>
 #include <algorithm>
 #include <cmath>
@@ -720,7 +720,7 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     // one token tile per CTA: balanced tiles of at most 256, rounded up to the MMA's N granule
     const int64_t t_tiles = (g.M + 255) / 256;
     int T = int(roundup((g.M + t_tiles - 1) / t_tiles, 16));
-    const bool split = g.K < 1024;
+    const bool split = g.K < 1024 || g.precise;
     int S = g.fmt == EMB_Q8_0   ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
             : g.fmt == EMB_Q4_0 ? (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T))
                                 : (split ? pick_stages<EMB_Q6_0, true>(T) : pick_stages<EMB_Q6_0, false>(T));

@@ -46,7 +46,9 @@ cudaError_t launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaS
 // rounded square root and reciprocal, then y = bf16(x * inv * gamma).
 constexpr int kNormThreads = 256;
 
-__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __restrict__ x,
+// x is read with coherent L2 loads (__ldcg): the previous launch wrote it while this grid
+// was already resident (programmatic dependent launch).
+__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x,
                                                                const float* __restrict__ gamma,
                                                                __nv_bfloat16* __restrict__ y,
                                                                int D, float eps) {
@@ -56,7 +58,7 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __re
     const float* xr = x + row * D;
     float ss = 0.0f;
     for (int i = threadIdx.x * 4; i < D; i += kNormThreads * 4) {
-        const float4 v = *reinterpret_cast<const float4*>(xr + i);
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(xr + i));
         ss = fmaf(v.x, v.x, ss);
         ss = fmaf(v.y, v.y, ss);
         ss = fmaf(v.z, v.z, ss);
@@ -77,7 +79,7 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __re
     const float inv = inv_s;
     __nv_bfloat16* yr = y + row * D;
     for (int i = threadIdx.x * 4; i < D; i += kNormThreads * 4) {
-        const float4 v = *reinterpret_cast<const float4*>(xr + i);
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(xr + i));
         const float4 g = *reinterpret_cast<const float4*>(gamma + i);
         const __nv_bfloat162 lo = __floats2bfloat162_rn(__fmul_rn(__fmul_rn(v.x, inv), g.x),
                                                         __fmul_rn(__fmul_rn(v.y, inv), g.y));
@@ -231,15 +233,17 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __grid_co
     const int64_t rA = row0 + warp * 16 + quad, rB = rA + 8;
     const int64_t offA = q_row(rA), offB = q_row(rB);
 
-    // Q fragments for the whole kernel (A operand, row-major 16 x D)
+    // Q fragments for the whole kernel (A operand, row-major 16 x D); coherent L2 loads,
+    // since the previous launch wrote Q while this grid was already resident
     uint32_t qf[KS][4];
+    auto ldq = [&](int64_t off) { return __ldcg(reinterpret_cast<const unsigned int*>(p.Q + off)); };
 #pragma unroll
     for (int ks = 0; ks < KS; ++ks) {
         const int c = ks * 16 + 2 * qc;
-        qf[ks][0] = offA >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offA + c) : 0u;
-        qf[ks][1] = offB >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offB + c) : 0u;
-        qf[ks][2] = offA >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offA + c + 8) : 0u;
-        qf[ks][3] = offB >= 0 ? *reinterpret_cast<const uint32_t*>(p.Q + offB + c + 8) : 0u;
+        qf[ks][0] = offA >= 0 ? ldq(offA + c) : 0u;
+        qf[ks][1] = offB >= 0 ? ldq(offB + c) : 0u;
+        qf[ks][2] = offA >= 0 ? ldq(offA + c + 8) : 0u;
+        qf[ks][3] = offB >= 0 ? ldq(offB + c + 8) : 0u;
     }
 
     // tile loader: 64 keys x D of keys and of values, 16-byte chunks, zero past the split

@@ -22,6 +22,25 @@ def test_every_declared_symbol_is_exported(L):
         assert hasattr(L, n), n
 
 
+def test_every_declaration_cites_its_passage():
+    """Every EMB_API declaration of include/emb_qmm.h is preceded by its own comment that
+    names the paper passage (a Section or Table) the entry point serves."""
+    import re
+    with open(emb.HEADER_PATH) as fh:
+        text = fh.read()
+    body = text[text.index('extern "C" {'):]
+    decls = list(re.finditer(r"EMB_API\s+[\w\s\*]*?\b(emb_\w+)\s*\(", body))
+    assert len(decls) == len(emb.declared_symbols())
+    prev_end = 0
+    for d in decls:
+        between = body[prev_end:d.start()]
+        comments = re.findall(r"/\*.*?\*/", between, flags=re.S)
+        assert comments, f"{d.group(1)} has no comment of its own"
+        assert re.search(r"\b(Section|Table)\s+\d", comments[-1]), \
+            f"{d.group(1)}: its comment names no Section or Table"
+        prev_end = body.index(";", d.end()) + 1
+
+
 def test_no_undeclared_exports(L):
     import subprocess
     out = subprocess.run(["nm", "-D", "--defined-only", emb.LIB_PATH], capture_output=True,
@@ -150,6 +169,17 @@ def test_seq_workspace_is_zero_for_valid_chains(L):
     chain = _layers([(0, A, 128, 64, B, C), (1, A + (64 << 20), 256, 64, B, C + (1 << 20))])
     assert emb.emb_qlayer_seq_workspace(chain, 1) == 0
     assert emb.emb_qlayer_seq_workspace(chain, 816) == 0
+
+
+def test_precise_operand_flag(L):
+    """EMB_PRECISE_OPERAND may be OR-ed into any epilogue; other flag bits are rejected."""
+    for kind in range(5):
+        ok = _layers([(0, A, 128, 64, B, C, kind | emb.EMB_PRECISE_OPERAND)])
+        assert emb.emb_qlayer_seq_workspace(ok, 64) == 0
+    bad = _layers([(0, A, 128, 64, B, C, 0x200)])
+    assert L.emb_qlayer_seq_workspace(bad, 1, 64) == ctypes.c_size_t(-1).value
+    bad = _layers([(0, A, 128, 64, B, C, 5 | emb.EMB_PRECISE_OPERAND)])
+    assert L.emb_qlayer_seq_workspace(bad, 1, 64) == ctypes.c_size_t(-1).value
 
 
 def test_chain_create_rejects(L):
