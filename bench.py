@@ -212,7 +212,8 @@ def build_chain(w: wl.Workload, device):
         n = resid_n.pop()
         resid = y_arena[:w.M * n * 4].view(torch.float32).view(w.M, n)
         yo = r256(w.M * n * 4)
-    specs, xs, ys, outs, images, x_bufs, y_bufs = [], [], [], [], {}, {}, {}
+    specs, xs, ys, outs, x_bufs, y_bufs = [], [], [], [], {}, {}
+    images = build_chain.images
     xo = 0
     for group in w.groups:
         K = group[0].K
@@ -229,7 +230,7 @@ def build_chain(w: wl.Workload, device):
             x_bufs[(group[0].name, K)] = X
         group_out = None
         for lin in group:
-            key = (lin.name, lin.N, lin.K, lin.seed)
+            key = (w.fmt, lin.name, lin.N, lin.K, lin.seed, lin.outliers)
             if key not in images:
                 W = wl.weight_torch(lin, device=device)
                 images[key] = emb.quantize(w.fmt, W)
@@ -256,6 +257,7 @@ def build_chain(w: wl.Workload, device):
 
 
 build_chain.arenas = {}   # id(specs) -> (activation arena, output arena)
+build_chain.images = {}   # (fmt, name, N, K, seed, outliers) -> packed device image, shared by chains
 
 
 def count_launches(specs) -> int:
@@ -447,17 +449,14 @@ def config_of(ws, args):
             "parallelism": f"replica x{int(os.environ.get('WORLD_SIZE', '1'))}"}
 
 
-def run_ours(args):
+def measure_workload(name, ws, args, dev, dist, steps, warmup, e2e_steps, clocks=True):
+    """Build the workload's chains, record each once, and time `steps` passes (after
+    `warmup`) with CUDA events on the launching stream: per pass and per chain. Returns the
+    measured figures: value / unit (the workload's metric), roofline of the dominant chain
+    and of every format, e2e through the public API, clocks."""
     import torch
     import paper_2607_02501_gb300 as emb
-    rank, world, local = dist_env()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    dist = init_dist(world, "nccl")
-    emb.lib()
-    ws = WORKLOADS[args.workload]()
-    if args.layers:
-        ws = [truncate(w, args.layers) for w in ws]
+    world = dist.get_world_size() if dist is not None else 1
     chains = []
     for w in ws:
         specs, xs, ys = build_chain(w, dev)
@@ -471,21 +470,21 @@ def run_ours(args):
     peaks = load_peaks()
     ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
     roof_tensor = all(w.flops() / w.algorithmic_bytes() >= ridge for w in ws)
-    # warm-up
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         for c in chains:
             for _ in range(c["w"].repeats):
                 c["graph"].replay()
     torch.cuda.synchronize()
     assert emb.emb_device_status() == emb.EMB_OK
 
-    sampler = ClockSampler(local)
-    sampler.start()
+    sampler = ClockSampler(torch.cuda.current_device()) if clocks else None
+    if sampler:
+        sampler.start()
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(chains) + 1)]
-          for _ in range(args.steps)]
+          for _ in range(steps)]
     barrier(dist)
     torch.cuda.synchronize()
-    for i in range(args.steps):
+    for i in range(steps):
         ev[i][0].record()
         for j, c in enumerate(chains):
             for _ in range(c["w"].repeats):
@@ -493,65 +492,132 @@ def run_ours(args):
             ev[i][j + 1].record()
     torch.cuda.synchronize()
     barrier(dist)
-    clocks = sampler.stop()
+    clock = sampler.stop() if sampler else None
     total_ms = ev[0][0].elapsed_time(ev[-1][-1])
-    chain_ms = [sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(args.steps))
+    chain_ms = [sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(steps))
                 for j in range(len(chains))]
-    per_step = step_stats([ev[i][0].elapsed_time(ev[i][-1]) for i in range(args.steps)])
+    per_step = step_stats([ev[i][0].elapsed_time(ev[i][-1]) for i in range(steps)])
     assert emb.emb_device_status() == emb.EMB_OK
     max_ms = max_over_ranks(total_ms, dist, dev)
 
     step_bytes = sum(c["bytes"] * c["w"].repeats for c in chains)
     step_flops = sum(c["flops"] * c["w"].repeats for c in chains)
     if tensor_bound:
-        value = world * step_flops * args.steps / (max_ms / 1e3) / 1e12
+        value = world * step_flops * steps / (max_ms / 1e3) / 1e12
         unit = "TFLOP/s"
     else:
-        value = world * step_bytes * args.steps / (max_ms / 1e3) / 1e9
+        value = world * step_bytes * steps / (max_ms / 1e3) / 1e9
         unit = "GB/s"
 
+    def roofline(k):
+        """Roofline of chain k: its algorithmic bytes (or flops) per launch over its
+        average launch duration in the timed region."""
+        c = chains[k]
+        launches = c["launches"] * c["w"].repeats * steps
+        per_launch_ms = chain_ms[k] / launches
+        if roof_tensor:
+            achieved = c["flops"] * c["w"].repeats * steps / launches / (per_launch_ms / 1e3) / 1e12
+            roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops_sustained"],
+                    "unit": "TFLOP/s", "peak_source": f"{peaks['source']} bf16 dense (sustained)"}
+        else:
+            achieved = c["bytes"] * c["w"].repeats * steps / launches / (per_launch_ms / 1e3) / 1e9
+            roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "peak_source": f"{peaks['source']} HBM copy bandwidth"}
+        roof["frac"] = roof["achieved"] / roof["peak"]
+        roof["traffic"] = kernel_traffic(name, c["w"])
+        roof["kernel"] = ("GEMV (gemv_staged_kernel + gemv_kernel + gemv_q4_mma_kernel)" if c["w"].M <= 4
+                          else "gemm_tc_kernel") + f" <{wl.FMT_NAMES[c['w'].fmt]}>"
+        roof["launches_per_step"] = c["launches"] * c["w"].repeats
+        roof["per_launch_us"] = per_launch_ms * 1e3
+        return roof
+
     # dominant kernel family: the chain that takes the most time
-    j = max(range(len(chains)), key=lambda k: chain_ms[k])
-    c = chains[j]
-    launches = c["launches"] * c["w"].repeats * args.steps
-    per_launch_ms = chain_ms[j] / launches
-    if roof_tensor:
-        achieved = c["flops"] * c["w"].repeats * args.steps / launches / (per_launch_ms / 1e3) / 1e12
-        roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops_sustained"],
-                "unit": "TFLOP/s", "peak_source": f"{peaks['source']} bf16 dense (sustained)"}
-    else:
-        achieved = c["bytes"] * c["w"].repeats * args.steps / launches / (per_launch_ms / 1e3) / 1e9
-        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "peak_source": f"{peaks['source']} HBM copy bandwidth"}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = kernel_traffic(args.workload, c["w"])
-    roof["kernel"] = ("GEMV (gemv_staged_kernel + gemv_kernel + gemv_q4_mma_kernel)" if c["w"].M <= 4
-                      else "gemm_tc_kernel") + f" <{wl.FMT_NAMES[c['w'].fmt]}>"
-    roof["launches_per_step"] = c["launches"] * c["w"].repeats
-    roof["per_launch_us"] = per_launch_ms * 1e3
+    dominant = max(range(len(chains)), key=lambda k: chain_ms[k])
+    per_format = {}
+    for k, cc in enumerate(chains):
+        per_format[wl.FMT_NAMES[cc["w"].fmt]] = {
+            "ms_per_step": chain_ms[k] / steps,
+            unit: (cc["flops"] if tensor_bound else cc["bytes"]) * cc["w"].repeats * steps
+            / (chain_ms[k] / 1e3) / (1e12 if tensor_bound else 1e9),
+            "roofline": roofline(k)}
+    e2e = measure_e2e(chains, e2e_steps, dev, dist, tensor_bound)
+    return {"chains": chains, "ws": ws, "value": value, "unit": unit, "max_ms": max_ms,
+            "ms_per_step": max_ms / steps, "step_ms": per_step, "roofline": roofline(dominant),
+            "per_format": per_format, "e2e": e2e, "clocks": clock, "tensor_bound": tensor_bound,
+            "gpu_launches": sum(cc["launches"] * cc["w"].repeats for cc in chains) * steps}
 
-    e2e = measure_e2e(chains, args, dev, dist, tensor_bound)
-    isolated = isolated_launch_us(chains[0]["specs"], ws[0].M) if args.workload == "single_linear" else None
 
-    gpu_launches = sum(cc["launches"] * cc["w"].repeats for cc in chains) * args.steps
-    line = {"metric": metric_name(ws), "value": value, "unit": unit, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": max_ms / args.steps,
+# Every configuration the bench reports beside its headline (one entry per configuration of
+# the workload list: the single linear, the 2B decoder at M = 1 (the headline itself), the
+# action expert's denoising loop at M = 50, the 2B prefill at M = 816 and the vision tower
+# at M = 768, the 7B backbone at M = 1 and M = 280).
+CONFIG_WORKLOADS = [("1_single_linear_q8_0_m1", "single_linear"),
+                    ("2_gemma2b_decode_m1", "gemma2b_decode"),
+                    ("3_action_expert_m50", "action_expert"),
+                    ("4_gemma2b_prefill_m816", "gemma2b_prefill"),
+                    ("4_vit_m768", "vit"),
+                    ("5_llama7b_decode_m1", "llama7b_decode"),
+                    ("5_llama7b_prefill_m280", "llama7b_prefill")]
+
+
+def config_entry(m):
+    """The per-configuration summary of a measure_workload result."""
+    return {"value": m["value"], "unit": m["unit"], "ms_per_step": m["ms_per_step"],
+            "roofline": {k: m["roofline"][k] for k in ("bound", "achieved", "peak", "unit", "frac",
+                                                      "traffic", "kernel")},
+            "per_format": {f: {"ms_per_step": v["ms_per_step"], m["unit"]: v[m["unit"]],
+                               "roofline": {k: v["roofline"][k] for k in ("achieved", "peak", "frac",
+                                                                         "traffic")}}
+                           for f, v in m["per_format"].items()},
+            "e2e": {k: m["e2e"][k] for k in ("value", "unit", "h2d_bytes_per_step", "d2h_bytes_per_step")},
+            "formats": [wl.FMT_NAMES[w.fmt] for w in m["ws"]], "M": m["ws"][0].M}
+
+
+def run_ours(args):
+    import torch
+    import paper_2607_02501_gb300 as emb
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = init_dist(world, "nccl")
+    emb.lib()
+    ws = WORKLOADS[args.workload]()
+    if args.layers:
+        ws = [truncate(w, args.layers) for w in ws]
+    m = measure_workload(args.workload, ws, args, dev, dist, args.steps, args.warmup,
+                         max(1, min(args.steps, 200)))
+    isolated = isolated_launch_us(m["chains"][0]["specs"], ws[0].M) if args.workload == "single_linear" else None
+    line = {"metric": metric_name(ws), "value": m["value"], "unit": m["unit"], "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": m["ms_per_step"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "bf16" if tensor_bound else "f32", "data": "synthetic",
-            "config": config_of(ws, args), "roofline": roof, "e2e": e2e, "clocks": clocks,
-            "gpu_launches": gpu_launches,
-            "per_format": {wl.FMT_NAMES[cc["w"].fmt]: {
-                "ms_per_step": chain_ms[k] / args.steps,
-                ("TFLOP/s" if tensor_bound else "GB/s"):
-                    (cc["flops"] if tensor_bound else cc["bytes"]) * cc["w"].repeats * args.steps
-                    / (chain_ms[k] / 1e3) / (1e12 if tensor_bound else 1e9)}
-                for k, cc in enumerate(chains)}}
-    line["step_ms"] = per_step
+            "dtype": "bf16" if m["tensor_bound"] else "f32", "data": "synthetic",
+            "config": config_of(ws, args), "roofline": m["roofline"], "e2e": m["e2e"],
+            "clocks": m["clocks"], "gpu_launches": m["gpu_launches"],
+            "per_format": {f: {"ms_per_step": v["ms_per_step"], m["unit"]: v[m["unit"]],
+                               "roofline": v["roofline"]} for f, v in m["per_format"].items()}}
+    line["step_ms"] = m["step_ms"]
     if isolated is not None:
         line["isolated_launch_us"] = isolated
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         torch.cuda.synchronize()
         line["cpu_baseline"] = cpu_baseline(ws)
+    if world == 1 and not args.no_configs and args.workload == "gemma2b_decode" and not args.layers:
+        # every configuration, a few timed passes each (after the headline's timed region)
+        cfg_steps = max(3, min(args.steps, 10))
+        configs = {}
+        for key, wname in CONFIG_WORKLOADS:
+            if wname == args.workload:
+                configs[key] = config_entry(m)
+                continue
+            cm = measure_workload(wname, WORKLOADS[wname](), args, dev, dist, cfg_steps, 3,
+                                  max(1, min(cfg_steps, 5)), clocks=False)
+            configs[key] = config_entry(cm)
+            configs[key]["steps"] = cfg_steps
+            for c in cm["chains"]:
+                c["graph"].close()
+                build_chain.arenas.pop(id(c["specs"]), None)
+            del cm
+        line["configs"] = configs
     if rank == 0:
         print(json.dumps(line))
     if dist is not None:
@@ -603,7 +669,7 @@ def kernel_traffic(workload, w):
         return None
 
 
-def measure_e2e(chains, args, dev, dist, tensor_bound):
+def measure_e2e(chains, steps, dev, dist, tensor_bound):
     """Same metric through the public call a user makes: per step, copy every layer's
     activations from pinned host memory, run emb_qlayer_seq for each format, copy every
     output back, synchronise."""
@@ -614,7 +680,6 @@ def measure_e2e(chains, args, dev, dist, tensor_bound):
     host_y = [torch.empty(ya.shape, dtype=ya.dtype).pin_memory() for _, ya in arenas]
     h2d = sum(x.numel() * x.element_size() for x in host_x)   # the bytes each step copies
     d2h = sum(y.numel() * y.element_size() for y in host_y)
-    steps = max(1, min(args.steps, 200))
 
     def one_step():
         # per chain: every activation in (one copy of the arena), the recorded chain
@@ -924,6 +989,8 @@ def main(argv=None):
     ap.add_argument("--workload", choices=sorted(list(WORKLOADS) + list(LAYER_LOOPS)),
                     default="gemma2b_decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-configuration section of the default line")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first L layers (small cases for ncu captures; "
                          "a number taken this way is not the workload's bench value)")

@@ -18,8 +18,9 @@
 // The first two dequantise in registers with exact integer->float "magic number"
 // conversions followed by packed fp32x2 FMAs (FFMA2). Every reduction runs in a fixed
 // order, so results are deterministic. Weights are fetched before griddepcontrol.wait (they never depend
-// on an earlier launch) with non-coherent streaming loads; X is read (coherent loads at L2:
-// the previous launch may have just written it) and Y written only after it.
+// on an earlier launch) with non-coherent streaming loads; X is read with ordinary
+// (coherent, L1-cached) loads and Y written only after it: the previous launch may have
+// just written X, and after griddepcontrol.wait its writes are visible to ordinary loads.
 // Up to kMaxGroup matrices that read the same X (q/k/v or gate/up) share one launch.
 #include <mutex>
 
@@ -145,7 +146,7 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
             const uint4* xp = reinterpret_cast<const uint4*>(p.X + int64_t(m0) * p.K + int64_t(uk) * UW);
 #pragma unroll
             for (int v = 0; v < UW / 8; ++v) {
-                const uint4 hx = __ldcg(xp + v);
+                const uint4 hx = xp[v];
                 x[8 * v + 0] = lo_bf16(hx.x); x[8 * v + 1] = hi_bf16(hx.x);
                 x[8 * v + 2] = lo_bf16(hx.y); x[8 * v + 3] = hi_bf16(hx.y);
                 x[8 * v + 4] = lo_bf16(hx.z); x[8 * v + 5] = hi_bf16(hx.z);
@@ -175,7 +176,7 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
             const uint4* xp = reinterpret_cast<const uint4*>(p.X + int64_t(m) * p.K + int64_t(u) * UW);
 #pragma unroll
             for (int v = 0; v < UW / 8; ++v) {
-                const uint4 h = __ldcg(xp + v);
+                const uint4 h = xp[v];
                 x[8 * v + 0] = lo_bf16(h.x); x[8 * v + 1] = hi_bf16(h.x);
                 x[8 * v + 2] = lo_bf16(h.y); x[8 * v + 3] = hi_bf16(h.y);
                 x[8 * v + 4] = lo_bf16(h.z); x[8 * v + 5] = hi_bf16(h.z);

@@ -46,8 +46,9 @@ cudaError_t launch_pdl(const void* fn, dim3 grid, dim3 block, size_t smem, cudaS
 // rounded square root and reciprocal, then y = bf16(x * inv * gamma).
 constexpr int kNormThreads = 256;
 
-// x is read with coherent L2 loads (__ldcg): the previous launch wrote it while this grid
-// was already resident (programmatic dependent launch).
+// x is read with ordinary loads (not the read-only path): the previous launch wrote it
+// while this grid was already resident (programmatic dependent launch); its writes are
+// visible to ordinary loads after griddepcontrol.wait.
 __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x,
                                                                const float* __restrict__ gamma,
                                                                __nv_bfloat16* __restrict__ y,
@@ -58,7 +59,7 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x,
     const float* xr = x + row * D;
     float ss = 0.0f;
     for (int i = threadIdx.x * 4; i < D; i += kNormThreads * 4) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(xr + i));
+        const float4 v = *reinterpret_cast<const float4*>(xr + i);
         ss = fmaf(v.x, v.x, ss);
         ss = fmaf(v.y, v.y, ss);
         ss = fmaf(v.z, v.z, ss);
@@ -79,7 +80,7 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x,
     const float inv = inv_s;
     __nv_bfloat16* yr = y + row * D;
     for (int i = threadIdx.x * 4; i < D; i += kNormThreads * 4) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(xr + i));
+        const float4 v = *reinterpret_cast<const float4*>(xr + i);
         const float4 g = *reinterpret_cast<const float4*>(gamma + i);
         const __nv_bfloat162 lo = __floats2bfloat162_rn(__fmul_rn(__fmul_rn(v.x, inv), g.x),
                                                         __fmul_rn(__fmul_rn(v.y, inv), g.y));
@@ -233,10 +234,10 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __grid_co
     const int64_t rA = row0 + warp * 16 + quad, rB = rA + 8;
     const int64_t offA = q_row(rA), offB = q_row(rB);
 
-    // Q fragments for the whole kernel (A operand, row-major 16 x D); coherent L2 loads,
-    // since the previous launch wrote Q while this grid was already resident
+    // Q fragments for the whole kernel (A operand, row-major 16 x D); ordinary loads, since
+    // the previous launch wrote Q while this grid was already resident
     uint32_t qf[KS][4];
-    auto ldq = [&](int64_t off) { return __ldcg(reinterpret_cast<const unsigned int*>(p.Q + off)); };
+    auto ldq = [&](int64_t off) { return *reinterpret_cast<const uint32_t*>(p.Q + off); };
 #pragma unroll
     for (int ks = 0; ks < KS; ++ks) {
         const int c = ks * 16 + 2 * qc;

@@ -64,3 +64,16 @@ def test_distinct_bytes_count_reused_weights_once():
     import workloads as wl
     w = wl.action_expert_fused()
     assert bench.distinct_weight_bytes([w]) * 10 == w.weight_bytes()
+
+
+def test_default_line_covers_every_configuration():
+    """The default run's `configs` section has one entry per workload configuration (the
+    single linear, the 2B decoder at M = 1, the action expert at M = 50, the 2B prefill and
+    the vision tower, the 7B backbone at M = 1 and M = 280), each a bench workload."""
+    keys = [k for k, _ in bench.CONFIG_WORKLOADS]
+    assert sorted({k.split("_")[0] for k in keys}) == ["1", "2", "3", "4", "5"]
+    for _, name in bench.CONFIG_WORKLOADS:
+        assert name in bench.WORKLOADS
+    Ms = {name: bench.WORKLOADS[name]()[0].M for _, name in bench.CONFIG_WORKLOADS}
+    assert Ms == {"single_linear": 1, "gemma2b_decode": 1, "action_expert": 50,
+                  "gemma2b_prefill": 816, "vit": 768, "llama7b_decode": 1, "llama7b_prefill": 280}
