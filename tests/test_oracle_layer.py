@@ -248,8 +248,11 @@ def _fp32_attention_model(Q, K, V, H, Hk, d, scale, splits, block):
     return out
 
 
-@pytest.mark.parametrize("n0,n1,splits", [(816, 50, 8), (100, 7, 2), (5, 0, 1)])
-def test_attention_bound_covers_an_fp32_model(n0, n1, splits):
+@pytest.mark.parametrize("n0,n1,splits,block", [(816, 50, 8, 64), (816, 50, 1, 1), (816, 50, 16, 7),
+                                                (100, 7, 2, 64), (100, 7, 3, 1), (5, 0, 1, 64)])
+def test_attention_bound_covers_an_fp32_model(n0, n1, splits, block):
+    """The bound holds for an fp32 online softmax whatever its key splits and key blocks
+    (down to a rescale after every key): it depends on the sizes and inputs only."""
     H, Hk, d = 8, 1, 128
     M = 3
     Q, K0, V0, K1, V1 = (_rand((M, H * d)), _rand((n0, Hk * d)), _rand((n0, Hk * d)),
@@ -257,5 +260,5 @@ def test_attention_bound_covers_an_fp32_model(n0, n1, splits):
     scale = 1.0 / math.sqrt(d)
     ref, bound = oracle.attention_reference(Q, K0, V0, K1, V1, H, Hk, d, scale)
     model = _fp32_attention_model(Q, np.concatenate([K0, K1]), np.concatenate([V0, V1]),
-                                  H, Hk, d, scale, splits, 64)
+                                  H, Hk, d, scale, splits, block)
     assert (np.abs(model - ref) <= bound).all()
