@@ -718,13 +718,47 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     int tiles = 0;
     for (int i = 0; i < g.n_mats; ++i) tiles += int((g.mats[i].N + kBN - 1) / kBN);
     // one token tile per CTA: balanced tiles of at most 256, rounded up to the MMA's N granule
-    const int64_t t_tiles = (g.M + 255) / 256;
+    int64_t t_tiles = (g.M + 255) / 256;
     int T = int(roundup((g.M + t_tiles - 1) / t_tiles, 16));
     const bool split = g.K < 1024 || g.precise;
     int S = g.fmt == EMB_Q8_0   ? (split ? pick_stages<EMB_Q8_0, true>(T) : pick_stages<EMB_Q8_0, false>(T))
             : g.fmt == EMB_Q4_0 ? (split ? pick_stages<EMB_Q4_0, true>(T) : pick_stages<EMB_Q4_0, false>(T))
                                 : (split ? pick_stages<EMB_Q6_0, true>(T) : pick_stages<EMB_Q6_0, false>(T));
     int splits = pick_splits(int64_t(t_tiles) * tiles, T, g.K, S, split);
+    // Prefill shapes whose weight tiles x token tiles leave SMs idle (narrow layers: the
+    // vision tower's 1152-wide ones give 9-36 weight tiles) may take more, smaller token
+    // tiles: per the cycle model below (per 64-k step the larger of the dequantisation,
+    // ~1050 cycles, and the MMA work, ~5.2 cycles per token; ~3900 per CTA; times the
+    // waves), up to three more tiles when that is at least 3 % faster. ViT M = 768: four
+    // tiles of 192 instead of three of 256 (qkv 81 -> 108 CTAs, fc1 108 -> 144).
+    if (!split && g.M >= 256) {
+        const int sms = sm_count();
+        if (sms > 0) {
+            const double nk = double((g.K + kKC - 1) / kKC);
+            auto cost = [&](int64_t tt, int Tc, int sp) {
+                return double((tt * tiles * sp + sms - 1) / sms) *
+                       (std::ceil(nk / sp) * std::max(1050.0, 5.2 * Tc) + 3900.0);
+            };
+            double best = cost(t_tiles, T, splits);
+            const int64_t t0 = t_tiles;
+            for (int64_t tt = t0 + 1; tt <= t0 + 3; ++tt) {
+                const int Tc = int(roundup((g.M + tt - 1) / tt, 16));
+                if (Tc < 64) break;
+                const int Sc = g.fmt == EMB_Q8_0 ? pick_stages<EMB_Q8_0, false>(Tc)
+                               : g.fmt == EMB_Q4_0 ? pick_stages<EMB_Q4_0, false>(Tc)
+                                                   : pick_stages<EMB_Q6_0, false>(Tc);
+                const int spc = pick_splits(tt * tiles, Tc, g.K, Sc, false);
+                const double c = cost(tt, Tc, spc);
+                if (c < 0.97 * best) {
+                    best = c;
+                    t_tiles = tt;
+                    T = Tc;
+                    S = Sc;
+                    splits = spc;
+                }
+            }
+        }
+    }
     int P = 1, grid_x = int(t_tiles);
     // Two token tiles per CTA halve the dequantisation per token (each A tile feeds the MMAs
     // of both). Time model in cycles, fitted to GB300 measurements of both formats: per
