@@ -79,6 +79,8 @@ struct GemmParams {
     int32_t a_gap0;                        // P = 2: TMEM column of the first A stage after tile 0's
     int32_t a_per_gap;                     //   accumulator, and A stages per gap (see pick_stages_pair)
     uint32_t tmem_cols;
+    int32_t persist;                       // 1: CTAs loop over items (no K split)
+    int32_t n_tt, n_items;                 // persistent: token tiles per weight tile, items
     int* status;
 };
 
@@ -169,7 +171,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint64_t* a_full = x_full + S;
     uint64_t* ax_empty = a_full + S;
     uint64_t* acc_full = ax_empty + S;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+    uint64_t* acc_empty = acc_full + 1;  // the epilogue warps have read the accumulator
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     volatile int* mma_stop = abort_flag + 1;  // set by the waiter warp when a wait gave up
     // split-K partial tile [T][128] fp32 (token-major): reuses the X ring once every MMA
@@ -177,21 +180,40 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     float* part = reinterpret_cast<float*>(x_ring);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile = blockIdx.y;
-    int g = 0;
-#pragma unroll
-    for (int i = 1; i < kMaxGroup; ++i)
-        if (i < p.n_mats && tile >= p.tile0[i]) g = i;
-    const int n0 = (tile - p.tile0[g]) * kBN;
-    const int m0 = blockIdx.x * P * T;  // first token of the CTA's first token tile
-    const int N = p.N[g], M = p.M, K = p.K;
-    // this CTA's K range: split-K over raw stages of 256
+    const int M = p.M, K = p.K;
+    // this CTA's K range: split-K over raw stages of 256 (the same for all of its items)
     const int splits = gridDim.z, split = blockIdx.z;
     const int nr_all = (K + kKR - 1) / kKR, nk_all = (K + kKC - 1) / kKC;
     const int rs0 = split * nr_all / splits, rs1 = (split + 1) * nr_all / splits;
     const int nr = rs1 - rs0;
     const int ks0 = rs0 * kStepsPerRaw;
     const int nk = min(rs1 * kStepsPerRaw, nk_all) - ks0;
+    // Work items (weight tile, token tile). Without p.persist each CTA has one: grid x =
+    // token tile, y = weight tile, z = K split. With p.persist (no K split) CTA c takes items
+    // c, c + gridDim.x, ... in the order of token tiles within weight tiles, so the CTAs at
+    // work on a weight tile at one time read it once from HBM and then from L2. Rings and
+    // barrier phases run on across items; the next item's codes and activations stream in
+    // while the current item's epilogue drains the accumulator.
+    const bool persist = p.persist != 0;
+    const int first_item = persist ? int(blockIdx.x) : 0;
+    const int item_stride = persist ? int(gridDim.x) : 1;
+    const int n_items = persist ? p.n_items : 1;
+    struct Item {
+        int g, n0, m0, N;
+    };
+    auto item_at = [&](int it) {
+        const int tt = persist ? it % p.n_tt : int(blockIdx.x);
+        const int tile = persist ? it / p.n_tt : int(blockIdx.y);
+        Item r;
+        r.g = 0;
+#pragma unroll
+        for (int i = 1; i < kMaxGroup; ++i)
+            if (i < p.n_mats && tile >= p.tile0[i]) r.g = i;
+        r.n0 = (tile - p.tile0[r.g]) * kBN;
+        r.m0 = tt * P * T;  // first token of the item's first token tile
+        r.N = p.N[r.g];
+        return r;
+    };
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kRawStages; ++i) {
@@ -204,13 +226,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             ptx::mbar_init(&ax_empty[i], 1);
         }
         ptx::mbar_init(acc_full, 1);
+        ptx::mbar_init(acc_empty, kDeqWarps);
         *abort_flag = 0;
         *mma_stop = 0;
         ptx::fence_mbar_init();
         ptx::prefetch_tmap(&p.x_map);
-        ptx::prefetch_tmap(&p.codes_map[g]);
-        ptx::prefetch_tmap(&p.scales_map[g]);
-        if constexpr (FMT == EMB_Q6_0) ptx::prefetch_tmap(&p.high_map[g]);
+        for (int i = 0; i < p.n_mats; ++i) {
+            ptx::prefetch_tmap(&p.codes_map[i]);
+            ptx::prefetch_tmap(&p.scales_map[i]);
+            if constexpr (FMT == EMB_Q6_0) ptx::prefetch_tmap(&p.high_map[i]);
+        }
     }
     if (warp == 1) {
         ptx::tmem_alloc(tmem_slot, p.tmem_cols);
@@ -221,50 +246,68 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     ptx::griddep_launch_dependents();
+    int items_done = 0;  // this CTA's items started by its role (phase of acc_full / acc_empty)
 
     if (warp == 0) {
         if (lane == 0) {
             // ---------------------------------------------------------------- producer
             const uint64_t pol_w = ptx::policy_evict_first();
             const uint64_t pol_x = ptx::policy_evict_last();
-            auto issue_raw = [&](int r) {
-                const int slot = r % kRawStages;
-                const int rg = rs0 + r;  // raw stage index within the whole row
-                ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + RT::hbytes + kScaleTile);
+            int raw_issued = 0, x_issued = 0;  // over all items of the CTA
+            bool stop = false, waited = false;
+            for (int it = first_item; it < n_items && !stop; it += item_stride, ++items_done) {
+                const Item I = item_at(it);
+                const int rbase = items_done * nr, xbase = items_done * nk;
+                auto issue_raw = [&](int r) {  // raw stage r of this item (global rbase + r)
+                    const int rg_all = rbase + r;
+                    const int slot = rg_all % kRawStages;
+                    const int rg = rs0 + r;  // raw stage index within the whole row
+                    ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + RT::hbytes + kScaleTile);
 #pragma unroll
-                for (int pl = 0; pl < RT::planes; ++pl)
-                    ptx::tma_load_2d(r_ring + slot * RT::bytes + pl * kPlane, &p.codes_map[g],
-                                     &raw_full[slot], (rg * RT::planes + pl) * 128, n0, pol_w);
-                if constexpr (FMT == EMB_Q6_0)  // x = 64 bytes per raw stage: 16-byte aligned
-                    ptx::tma_load_2d(h_ring + slot * RT::hbytes, &p.high_map[g], &raw_full[slot],
-                                     rg * 64, n0, pol_w);
-                ptx::tma_load_2d(s_ring + slot * kScaleTile, &p.scales_map[g], &raw_full[slot],
-                                 rg * (kKR / kQBlock), n0, pol_w);
-            };
-            int raw_issued = 0, x_issued = 0;
-            for (; raw_issued < nr && raw_issued < kRawStages; ++raw_issued) issue_raw(raw_issued);
-            ptx::griddep_wait();  // X may be written by the previous launch
-            for (int i = 0; i < nk; ++i) {
-                if (i % kStepsPerRaw == 0) {
-                    const int r = i / kStepsPerRaw;
-                    if (r >= raw_issued) {
-                        if (!ptx::mbar_wait(&raw_empty[r % kRawStages], ((r / kRawStages) - 1) & 1,
-                                            abort_flag, p.status, kWaitLimitNs))
-                            break;
-                        issue_raw(r);
-                        ++raw_issued;
-                    }
+                    for (int pl = 0; pl < RT::planes; ++pl)
+                        ptx::tma_load_2d(r_ring + slot * RT::bytes + pl * kPlane, &p.codes_map[I.g],
+                                         &raw_full[slot], (rg * RT::planes + pl) * 128, I.n0, pol_w);
+                    if constexpr (FMT == EMB_Q6_0)  // x = 64 bytes per raw stage: 16-byte aligned
+                        ptx::tma_load_2d(h_ring + slot * RT::hbytes, &p.high_map[I.g], &raw_full[slot],
+                                         rg * 64, I.n0, pol_w);
+                    ptx::tma_load_2d(s_ring + slot * kScaleTile, &p.scales_map[I.g], &raw_full[slot],
+                                     rg * (kKR / kQBlock), I.n0, pol_w);
+                };
+                if (!waited) {
+                    // the first raw stages before griddepcontrol.wait: weights never depend on
+                    // the previous launch; X may be written by it
+                    for (; raw_issued < nr && raw_issued < kRawStages; ++raw_issued) issue_raw(raw_issued);
+                    ptx::griddep_wait();
+                    waited = true;
                 }
-                const int s = i % S;
-                if (i >= S && !ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
-                                              p.status, kWaitLimitNs))
-                    break;
-                ptx::mbar_arrive_expect_tx(&x_full[s], uint32_t(P * T) * 128u);
+                for (int i = 0; i < nk; ++i) {
+                    if (i % kStepsPerRaw == 0) {
+                        const int rg_all = rbase + i / kStepsPerRaw;
+                        if (rg_all >= raw_issued) {
+                            if (rg_all >= kRawStages &&
+                                !ptx::mbar_wait(&raw_empty[rg_all % kRawStages], ((rg_all / kRawStages) - 1) & 1,
+                                                abort_flag, p.status, kWaitLimitNs)) {
+                                stop = true;
+                                break;
+                            }
+                            issue_raw(i / kStepsPerRaw);
+                            ++raw_issued;
+                        }
+                    }
+                    const int xs = xbase + i;
+                    const int s = xs % S;
+                    if (xs >= S && !ptx::mbar_wait(&ax_empty[s], ((xs / S) - 1) & 1, abort_flag, p.status,
+                                                   kWaitLimitNs)) {
+                        stop = true;
+                        break;
+                    }
+                    ptx::mbar_arrive_expect_tx(&x_full[s], uint32_t(P * T) * 128u);
 #pragma unroll
-                for (int q = 0; q < P; ++q)  // a tile past M reads zeros (its outputs are not stored)
-                    ptx::tma_load_2d(x_ring + (s * P + q) * T * 128, &p.x_map, &x_full[s],
-                                     (ks0 + i) * kKC, m0 + q * T, pol_x);
-                ++x_issued;
+                    for (int q = 0; q < P; ++q)  // a tile past M reads zeros (its outputs are not stored)
+                        ptx::tma_load_2d(x_ring + (s * P + q) * T * 128, &p.x_map, &x_full[s],
+                                         (ks0 + i) * kKC, I.m0 + q * T, pol_x);
+                    ++x_issued;
+                }
             }
             // every issued copy must land before this CTA's shared memory can be released
             for (int r = raw_issued - 1; r >= 0 && r >= raw_issued - kRawStages; --r)
@@ -279,50 +322,73 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         // runs no mbarrier wait while MMAs are in flight (see kWaitWarp below).
         const uint32_t idesc = ptx::idesc_bf16_f32(kBN, T);
         const uint32_t x0 = ptx::smem_u32(x_ring);
-        for (int i = 0; i < nk; ++i) {
-            named_sync(1, 64);
-            if (*mma_stop) break;
-            if (lane == 0) {
-                const int s = i % S;
-                ptx::tc_fence_after();
-                const uint32_t a_tm = tmem + a_stage_col<P, SPLIT>(s, p.a_gap0, p.a_per_gap);
-#pragma unroll
-                for (int q = 0; q < P; ++q) {
-                    // token tile q: its own X tile and accumulator, the same A tile
-                    const uint32_t x_addr = x0 + (s * P + q) * T * 128;
-                    const uint32_t d_tm = tmem + uint32_t(q * kAccCols);
-#pragma unroll
-                    for (int k = 0; k < kKC / 16; ++k) {
-                        const uint64_t bdesc = ptx::smem_desc_sw128(x_addr + 32 * k);
-                        ptx::mma_bf16_ta(d_tm, a_tm + 8 * k, bdesc, idesc, (i | k) != 0);
-                        if constexpr (SPLIT) ptx::mma_bf16_ta(d_tm, a_tm + kACols + 8 * k, bdesc, idesc, 1u);
-                    }
+        bool stop = false;
+        int commits = 0;  // accumulator commits (one per finished item)
+        for (int it = first_item; it < n_items && !stop; it += item_stride, ++items_done) {
+            const int xbase = items_done * nk;
+            for (int i = 0; i < nk; ++i) {
+                named_sync(1, 64);
+                if (*mma_stop) {
+                    stop = true;
+                    break;
                 }
-                ptx::mma_commit(&ax_empty[s]);
+                if (lane == 0) {
+                    const int s = (xbase + i) % S;
+                    ptx::tc_fence_after();
+                    const uint32_t a_tm = tmem + a_stage_col<P, SPLIT>(s, p.a_gap0, p.a_per_gap);
+#pragma unroll
+                    for (int q = 0; q < P; ++q) {
+                        // token tile q: its own X tile and accumulator, the same A tile
+                        const uint32_t x_addr = x0 + (s * P + q) * T * 128;
+                        const uint32_t d_tm = tmem + uint32_t(q * kAccCols);
+#pragma unroll
+                        for (int k = 0; k < kKC / 16; ++k) {
+                            const uint64_t bdesc = ptx::smem_desc_sw128(x_addr + 32 * k);
+                            ptx::mma_bf16_ta(d_tm, a_tm + 8 * k, bdesc, idesc, (i | k) != 0);
+                            if constexpr (SPLIT) ptx::mma_bf16_ta(d_tm, a_tm + kACols + 8 * k, bdesc, idesc, 1u);
+                        }
+                    }
+                    ptx::mma_commit(&ax_empty[s]);
+                }
+                __syncwarp();
             }
+            // the item's accumulator is complete once every MMA issued so far has finished
+            if (stop) break;
+            if (lane == 0) ptx::mma_commit(acc_full);
+            ++commits;
             __syncwarp();
         }
-        if (lane == 0) {
-            ptx::mma_commit(acc_full);  // completes once every issued MMA has finished
-            ptx::mbar_wait(acc_full, 0, nullptr, p.status, kWaitLimitNs);
-        }
+        if (lane == 0 && commits > 0)  // the last item's MMAs finish before TMEM is freed
+            ptx::mbar_wait(acc_full, (commits - 1) & 1, nullptr, p.status, kWaitLimitNs);
     } else if (warp == kWaitWarp) {
         // ---------------------------------------------------------------- waiter
         // An mbarrier wait executed by the warp that issues tcgen05 MMAs is ordered behind
         // that warp's in-flight MMAs, which drains the tensor pipe at every step (measured
         // on GB300: 104 -> 330+ cycles per 128x208x16 MMA). This warp waits for step i's
-        // X tile and A tile and then releases the MMA warp through named barrier 1.
-        for (int i = 0; i < nk; ++i) {
-            const int s = i % S;
-            const uint32_t ph = (i / S) & 1;
-            if (lane == 0) {
-                const bool ok = ptx::mbar_wait(&x_full[s], ph, abort_flag, p.status, kWaitLimitNs) &&
-                                ptx::mbar_wait(&a_full[s], ph, abort_flag, p.status, kWaitLimitNs);
-                if (!ok) *mma_stop = 1;
+        // X tile and A tile (and, at an item's first step, for the previous item's epilogue
+        // to have read the accumulator) and then releases the MMA warp through named barrier 1.
+        bool stop = false;
+        for (int it = first_item; it < n_items && !stop; it += item_stride, ++items_done) {
+            const int xbase = items_done * nk;
+            for (int i = 0; i < nk; ++i) {
+                const int xs = xbase + i;
+                const int s = xs % S;
+                const uint32_t ph = (xs / S) & 1;
+                if (lane == 0) {
+                    bool ok = true;
+                    if (i == 0 && items_done > 0)
+                        ok = ptx::mbar_wait(acc_empty, (items_done - 1) & 1, abort_flag, p.status, kWaitLimitNs);
+                    ok = ok && ptx::mbar_wait(&x_full[s], ph, abort_flag, p.status, kWaitLimitNs) &&
+                         ptx::mbar_wait(&a_full[s], ph, abort_flag, p.status, kWaitLimitNs);
+                    if (!ok) *mma_stop = 1;
+                }
+                __syncwarp();
+                named_sync(1, 64);
+                if (*mma_stop) {
+                    stop = true;
+                    break;
+                }
             }
-            __syncwarp();
-            named_sync(1, 64);
-            if (*mma_stop) break;
         }
     } else if (warp < 2 + kDeqWarps) {
         // ---------------------------------------------------------------- dequant
@@ -333,178 +399,192 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         const uint32_t a_lane = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t(16 * h);
         const unsigned full = 0xffffffffu;
         bool ok = true;
-        // Software pipeline: step i's TMEM stores are completed (tcgen05.wait::st) and
-        // signalled only after step i+1 has been computed, so the store latency overlaps
-        // the next step's arithmetic instead of stalling this warp every step.
-        int pending = -1;  // A stage whose stores are in flight, not yet signalled
-        auto signal_pending = [&]() {
-            if (pending >= 0) {
-                ptx::tmem_st_wait();
-                ptx::tc_fence_before();  // the stores are ordered before the arrive
+        for (int it = first_item; it < n_items && ok; it += item_stride, ++items_done) {
+            const Item I = item_at(it);
+            const int rbase = items_done * nr, xbase = items_done * nk;
+            // Software pipeline: step i's TMEM stores are completed (tcgen05.wait::st) and
+            // signalled only after step i+1 has been computed, so the store latency overlaps
+            // the next step's arithmetic instead of stalling this warp every step.
+            int pending = -1;  // A stage whose stores are in flight, not yet signalled
+            auto signal_pending = [&]() {
+                if (pending >= 0) {
+                    ptx::tmem_st_wait();
+                    ptx::tc_fence_before();  // the stores are ordered before the arrive
+                    __syncwarp();
+                    if (lane == 0) ptx::mbar_arrive(&a_full[pending]);
+                    pending = -1;
+                }
+            };
+            for (int r = 0; r < nr && ok; ++r) {
+                const int rg_all = rbase + r;
+                const int rs = rg_all % kRawStages;
+                ok = __all_sync(full, ptx::mbar_wait(&raw_full[rs], (rg_all / kRawStages) & 1, abort_flag,
+                                                     p.status, kWaitLimitNs));
+                if (!ok) break;
+                const uint8_t* rbase_p = r_ring + rs * RT::bytes + t * 128;
+                const uint4 sv = lds128(s_ring + rs * kScaleTile + t * 16);
+                const uint32_t sw[4] = {sv.x, sv.y, sv.z, sv.w};
+                float d[4], nbd[4];  // scale of block 2j + h (word j, half h), j = 0..3
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const uint16_t hb = uint16_t((sw[j] >> (16 * h)) & 0xFFFFu);
+                    d[j] = __half2float(__ushort_as_half(hb));
+                    nbd[j] = -RT::bias * d[j];  // exact (see bytes_to_w)
+                }
+#pragma unroll
+                for (int j = 0; j < kStepsPerRaw; ++j) {
+                    const int i = r * kStepsPerRaw + j;
+                    if (i >= nk) break;
+                    const int xs = xbase + i;
+                    const int s = xs % S;
+                    const uint32_t a_dst = a_lane + a_stage_col<P, SPLIT>(s, p.a_gap0, p.a_per_gap);
+                    const int sx = t & 7;  // raw codes: 16-byte chunk c of row t lives at c ^ (t & 7)
+                    uint32_t va[16], vl[16];  // this thread's 16 columns of the hi (and lo) tile
+                    if constexpr (FMT == EMB_Q8_0) {
+                        // atom j: codes 64j..64j+63 of the raw stage = plane j/2, chunks 4(j%2)..+3;
+                        // this half: chunks 4(j%2)+2h, +1 (block 2j+h) -> output chunks 4h..4h+3
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int cc = 2 * h + e;
+                            const int c = (j & 1) * 4 + cc;
+                            const uint4 v = lds128(rbase_p + (j >> 1) * kPlane + ((c ^ sx) << 4));
+                            uint4 h0, l0, h1, l1;
+                            make_chunk<SPLIT>(v.x ^ 0x80808080u, v.y ^ 0x80808080u, d[j], nbd[j], h0, l0);
+                            make_chunk<SPLIT>(v.z ^ 0x80808080u, v.w ^ 0x80808080u, d[j], nbd[j], h1, l1);
+                            // output chunks 2cc, 2cc+1 (k = 16cc .. 16cc+15) -> columns 8e .. 8e+7
+                            const int q = 8 * e;
+                            va[q + 0] = h0.x; va[q + 1] = h0.y; va[q + 2] = h0.z; va[q + 3] = h0.w;
+                            va[q + 4] = h1.x; va[q + 5] = h1.y; va[q + 6] = h1.z; va[q + 7] = h1.w;
+                            if constexpr (SPLIT) {
+                                vl[q + 0] = l0.x; vl[q + 1] = l0.y; vl[q + 2] = l0.z; vl[q + 3] = l0.w;
+                                vl[q + 4] = l1.x; vl[q + 5] = l1.y; vl[q + 6] = l1.z; vl[q + 7] = l1.w;
+                            }
+                        }
+                    } else {
+                        // atom j: blocks 2j, 2j+1; this half: block 2j+h -> output chunks 4h..4h+3.
+                        // A block's byte i holds code i (low nibble) and code i+16 (high nibble).
+                        const int b = 2 * j + h;
+                        const uint4 v = lds128(rbase_p + ((b ^ sx) << 4));
+                        const uint32_t m = 0x0F0F0F0Fu;
+                        // Q4_0: the nibbles are the codes. Q6_0: OR in the high bits so that every
+                        // byte holds a whole code: high word (w & 1) >> 2(w >> 1) has the high bits
+                        // of low word w's codes at bits 0-1 (codes 4w+i) and 4-5 (codes 16+4w+i).
+                        uint32_t c0 = v.x & m, c1 = v.y & m, c2 = v.z & m, c3 = v.w & m;
+                        uint32_t e0 = (v.x >> 4) & m, e1 = (v.y >> 4) & m, e2 = (v.z >> 4) & m, e3 = (v.w >> 4) & m;
+                        if constexpr (FMT == EMB_Q6_0) {
+                            const uint2 hv = *reinterpret_cast<const uint2*>(h_ring + rs * RT::hbytes + t * 64 + b * 8);
+                            const uint32_t hw[4] = {hv.x, hv.y, hv.x >> 2, hv.y >> 2};
+                            c0 |= (hw[0] & 0x03030303u) << 4; e0 |= hw[0] & 0x30303030u;
+                            c1 |= (hw[1] & 0x03030303u) << 4; e1 |= hw[1] & 0x30303030u;
+                            c2 |= (hw[2] & 0x03030303u) << 4; e2 |= hw[2] & 0x30303030u;
+                            c3 |= (hw[3] & 0x03030303u) << 4; e3 |= hw[3] & 0x30303030u;
+                        }
+                        uint4 hh[4], ll[4];
+                        make_chunk<SPLIT>(c0, c1, d[j], nbd[j], hh[0], ll[0]);  // codes 0..7
+                        make_chunk<SPLIT>(c2, c3, d[j], nbd[j], hh[1], ll[1]);  // 8..15
+                        make_chunk<SPLIT>(e0, e1, d[j], nbd[j], hh[2], ll[2]);  // 16..23
+                        make_chunk<SPLIT>(e2, e3, d[j], nbd[j], hh[3], ll[3]);  // 24..31
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {  // output chunk 4h+q -> columns 4q .. 4q+3
+                            va[4 * q + 0] = hh[q].x; va[4 * q + 1] = hh[q].y;
+                            va[4 * q + 2] = hh[q].z; va[4 * q + 3] = hh[q].w;
+                            if constexpr (SPLIT) {
+                                vl[4 * q + 0] = ll[q].x; vl[4 * q + 1] = ll[q].y;
+                                vl[4 * q + 2] = ll[q].z; vl[4 * q + 3] = ll[q].w;
+                            }
+                        }
+                    }
+                    signal_pending();
+                    if (xs >= S) {
+                        ok = __all_sync(full, ptx::mbar_wait(&ax_empty[s], ((xs / S) - 1) & 1, abort_flag,
+                                                             p.status, kWaitLimitNs));
+                        if (!ok) break;
+                        ptx::tc_fence_after();  // the MMAs that read this A stage have completed
+                    }
+                    ptx::tmem_st_16(a_dst, va);
+                    if constexpr (SPLIT) ptx::tmem_st_16(a_dst + kACols, vl);
+                    pending = s;
+                }
+                if (!ok) break;
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(&a_full[pending]);
-                pending = -1;
+                if (lane == 0) ptx::mbar_arrive(&raw_empty[rs]);
             }
-        };
-        for (int r = 0; r < nr && ok; ++r) {
-            const int rs = r % kRawStages;
-            ok = __all_sync(full, ptx::mbar_wait(&raw_full[rs], (r / kRawStages) & 1, abort_flag,
-                                                 p.status, kWaitLimitNs));
-            if (!ok) break;
-            const uint8_t* rbase = r_ring + rs * RT::bytes + t * 128;
-            const uint4 sv = lds128(s_ring + rs * kScaleTile + t * 16);
-            const uint32_t sw[4] = {sv.x, sv.y, sv.z, sv.w};
-            float d[4], nbd[4];  // scale of block 2j + h (word j, half h), j = 0..3
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const uint16_t hb = uint16_t((sw[j] >> (16 * h)) & 0xFFFFu);
-                d[j] = __half2float(__ushort_as_half(hb));
-                nbd[j] = -RT::bias * d[j];  // exact (see bytes_to_w)
-            }
-#pragma unroll
-            for (int j = 0; j < kStepsPerRaw; ++j) {
-                const int i = r * kStepsPerRaw + j;
-                if (i >= nk) break;
-                const int s = i % S;
-                const uint32_t a_dst = a_lane + a_stage_col<P, SPLIT>(s, p.a_gap0, p.a_per_gap);
-                const int sx = t & 7;  // raw codes: 16-byte chunk c of row t lives at c ^ (t & 7)
-                uint32_t va[16], vl[16];  // this thread's 16 columns of the hi (and lo) tile
-                if constexpr (FMT == EMB_Q8_0) {
-                    // atom j: codes 64j..64j+63 of the raw stage = plane j/2, chunks 4(j%2)..+3;
-                    // this half: chunks 4(j%2)+2h, +1 (block 2j+h) -> output chunks 4h..4h+3
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int cc = 2 * h + e;
-                        const int c = (j & 1) * 4 + cc;
-                        const uint4 v = lds128(rbase + (j >> 1) * kPlane + ((c ^ sx) << 4));
-                        uint4 h0, l0, h1, l1;
-                        make_chunk<SPLIT>(v.x ^ 0x80808080u, v.y ^ 0x80808080u, d[j], nbd[j], h0, l0);
-                        make_chunk<SPLIT>(v.z ^ 0x80808080u, v.w ^ 0x80808080u, d[j], nbd[j], h1, l1);
-                        // output chunks 2cc, 2cc+1 (k = 16cc .. 16cc+15) -> columns 8e .. 8e+7
-                        const int q = 8 * e;
-                        va[q + 0] = h0.x; va[q + 1] = h0.y; va[q + 2] = h0.z; va[q + 3] = h0.w;
-                        va[q + 4] = h1.x; va[q + 5] = h1.y; va[q + 6] = h1.z; va[q + 7] = h1.w;
-                        if constexpr (SPLIT) {
-                            vl[q + 0] = l0.x; vl[q + 1] = l0.y; vl[q + 2] = l0.z; vl[q + 3] = l0.w;
-                            vl[q + 4] = l1.x; vl[q + 5] = l1.y; vl[q + 6] = l1.z; vl[q + 7] = l1.w;
-                        }
-                    }
-                } else {
-                    // atom j: blocks 2j, 2j+1; this half: block 2j+h -> output chunks 4h..4h+3.
-                    // A block's byte i holds code i (low nibble) and code i+16 (high nibble).
-                    const int b = 2 * j + h;
-                    const uint4 v = lds128(rbase + ((b ^ sx) << 4));
-                    const uint32_t m = 0x0F0F0F0Fu;
-                    // Q4_0: the nibbles are the codes. Q6_0: OR in the high bits so that every
-                    // byte holds a whole code: high word (w & 1) >> 2(w >> 1) has the high bits
-                    // of low word w's codes at bits 0-1 (codes 4w+i) and 4-5 (codes 16+4w+i).
-                    uint32_t c0 = v.x & m, c1 = v.y & m, c2 = v.z & m, c3 = v.w & m;
-                    uint32_t e0 = (v.x >> 4) & m, e1 = (v.y >> 4) & m, e2 = (v.z >> 4) & m, e3 = (v.w >> 4) & m;
-                    if constexpr (FMT == EMB_Q6_0) {
-                        const uint2 hv = *reinterpret_cast<const uint2*>(h_ring + rs * RT::hbytes + t * 64 + b * 8);
-                        const uint32_t hw[4] = {hv.x, hv.y, hv.x >> 2, hv.y >> 2};
-                        c0 |= (hw[0] & 0x03030303u) << 4; e0 |= hw[0] & 0x30303030u;
-                        c1 |= (hw[1] & 0x03030303u) << 4; e1 |= hw[1] & 0x30303030u;
-                        c2 |= (hw[2] & 0x03030303u) << 4; e2 |= hw[2] & 0x30303030u;
-                        c3 |= (hw[3] & 0x03030303u) << 4; e3 |= hw[3] & 0x30303030u;
-                    }
-                    uint4 hh[4], ll[4];
-                    make_chunk<SPLIT>(c0, c1, d[j], nbd[j], hh[0], ll[0]);  // codes 0..7
-                    make_chunk<SPLIT>(c2, c3, d[j], nbd[j], hh[1], ll[1]);  // 8..15
-                    make_chunk<SPLIT>(e0, e1, d[j], nbd[j], hh[2], ll[2]);  // 16..23
-                    make_chunk<SPLIT>(e2, e3, d[j], nbd[j], hh[3], ll[3]);  // 24..31
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {  // output chunk 4h+q -> columns 4q .. 4q+3
-                        va[4 * q + 0] = hh[q].x; va[4 * q + 1] = hh[q].y;
-                        va[4 * q + 2] = hh[q].z; va[4 * q + 3] = hh[q].w;
-                        if constexpr (SPLIT) {
-                            vl[4 * q + 0] = ll[q].x; vl[4 * q + 1] = ll[q].y;
-                            vl[4 * q + 2] = ll[q].z; vl[4 * q + 3] = ll[q].w;
-                        }
-                    }
-                }
-                signal_pending();
-                if (i >= S) {
-                    ok = __all_sync(full, ptx::mbar_wait(&ax_empty[s], ((i / S) - 1) & 1, abort_flag,
-                                                         p.status, kWaitLimitNs));
-                    if (!ok) break;
-                    ptx::tc_fence_after();  // the MMAs that read this A stage have completed
-                }
-                ptx::tmem_st_16(a_dst, va);
-                if constexpr (SPLIT) ptx::tmem_st_16(a_dst + kACols, vl);
-                pending = s;
-            }
-            if (!ok) break;
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&raw_empty[rs]);
-        }
-        if (ok) signal_pending();
-        ptx::tmem_st_wait();  // no store of this warp is left in flight, whatever happened
+            if (ok) signal_pending();
+            ptx::tmem_st_wait();  // no store of this warp is left in flight, whatever happened
 
-        // ---------------------------------------------------------------- epilogue
-        ptx::griddep_wait();  // Y may be read or written by the previous launch
-        ok = __all_sync(full, ok && ptx::mbar_wait(acc_full, 0, abort_flag, p.status, kWaitLimitNs));
-        if (ok) {
-            ptx::tc_fence_after();
-            // warps 2..9: TMEM lane quarter = warp % 4; the two warps of a quarter split the
-            // columns of one token tile, or (P = 2) take one token tile each
-            const int quarter = warp & 3, half = (warp - 2) >> 2;
-            const int csplit = ((T >> 1) + 15) & ~15;
-            const int tt = (P == 2) ? half : 0;  // token tile read by this warp
-            const int cbeg = (P == 2 || !half) ? 0 : csplit;
-            const int cend = (P == 2 || half) ? T : min(csplit, T);
-            const int row = quarter * 32 + lane;
-            const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16) + uint32_t(tt * kAccCols);
-            const int n = n0 + row;
-            const int mt = m0 + tt * T;  // first token of that tile
-            void* Y = p.Y[g];
-            const int epi = p.epi;
-            for (int c0 = cbeg; c0 < cend; c0 += 16) {
-                uint32_t v[16];
-                ptx::tmem_ld_16(taddr + uint32_t(c0), v);
-                ptx::tmem_ld_wait();
-                if (splits == 1) {
-                    if (epi >= EMB_EPI_GEGLU) {
-                        // gate row n (even lane) and up row n + 1 (the next lane): rows past N
-                        // hold zeros (their weights were read as zeros), so every lane shuffles
+            // ---------------------------------------------------------------- epilogue
+            ptx::griddep_wait();  // Y may be read or written by the previous launch
+            ok = __all_sync(full, ok && ptx::mbar_wait(acc_full, items_done & 1, abort_flag, p.status,
+                                                       kWaitLimitNs));
+            if (ok) {
+                ptx::tc_fence_after();
+                // warps 2..9: TMEM lane quarter = warp % 4; the two warps of a quarter split the
+                // columns of one token tile, or (P = 2) take one token tile each
+                const int quarter = warp & 3, half = (warp - 2) >> 2;
+                const int csplit = ((T >> 1) + 15) & ~15;
+                const int tt = (P == 2) ? half : 0;  // token tile read by this warp
+                const int cbeg = (P == 2 || !half) ? 0 : csplit;
+                const int cend = (P == 2 || half) ? T : min(csplit, T);
+                const int row = quarter * 32 + lane;
+                const uint32_t taddr = tmem + (uint32_t(quarter * 32) << 16) + uint32_t(tt * kAccCols);
+                const int n = I.n0 + row, N = I.N;
+                const int mt = I.m0 + tt * T;  // first token of that tile
+                void* Y = p.Y[I.g];
+                const int epi = p.epi;
+                for (int c0 = cbeg; c0 < cend; c0 += 16) {
+                    uint32_t v[16];
+                    ptx::tmem_ld_16(taddr + uint32_t(c0), v);
+                    ptx::tmem_ld_wait();
+                    if (splits == 1) {
+                        if (epi >= EMB_EPI_GEGLU) {
+                            // gate row n (even lane) and up row n + 1 (the next lane): rows past N
+                            // hold zeros (their weights were read as zeros), so every lane shuffles
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            const float up = __shfl_down_sync(0xffffffffu, __uint_as_float(v[e]), 1);
-                            const int m = mt + c0 + e;
-                            if ((lane & 1) == 0 && n < N && m < M)
-                                epi_store_gated(epi, Y, m, n, N, __uint_as_float(v[e]), up);
+                            for (int e = 0; e < 16; ++e) {
+                                const float up = __shfl_down_sync(0xffffffffu, __uint_as_float(v[e]), 1);
+                                const int m = mt + c0 + e;
+                                if ((lane & 1) == 0 && n < N && m < M)
+                                    epi_store_gated(epi, Y, m, n, N, __uint_as_float(v[e]), up);
+                            }
+                        } else if (epi == EMB_EPI_ADD && n < N) {
+                            // reads four at a time ahead of their stores: a read after a store to
+                            // the same buffer would otherwise wait for that store
+                            float* y = reinterpret_cast<float*>(Y);
+#pragma unroll
+                            for (int e0 = 0; e0 < 16; e0 += 4) {
+                                float old[4];
+#pragma unroll
+                                for (int e = 0; e < 4; ++e)
+                                    old[e] = (mt + c0 + e0 + e < M) ? y[int64_t(mt + c0 + e0 + e) * N + n] : 0.0f;
+#pragma unroll
+                                for (int e = 0; e < 4; ++e)
+                                    if (mt + c0 + e0 + e < M)
+                                        y[int64_t(mt + c0 + e0 + e) * N + n] =
+                                            __fadd_rn(old[e], __uint_as_float(v[e0 + e]));
+                            }
+                        } else if (n < N) {
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                const int m = mt + c0 + e;
+                                if (m < M) epi_store(epi, Y, m, n, N, __uint_as_float(v[e]));
+                            }
                         }
-                    } else if (epi == EMB_EPI_ADD && n < N) {
-                        // reads four at a time ahead of their stores: a read after a store to
-                        // the same buffer would otherwise wait for that store
-                        float* y = reinterpret_cast<float*>(Y);
+                    } else {
+                        // token-major partial tile part[m][row] (a warp writes 32 consecutive rows)
 #pragma unroll
-                        for (int e0 = 0; e0 < 16; e0 += 4) {
-                            float old[4];
-#pragma unroll
-                            for (int e = 0; e < 4; ++e)
-                                old[e] = (mt + c0 + e0 + e < M) ? y[int64_t(mt + c0 + e0 + e) * N + n] : 0.0f;
-#pragma unroll
-                            for (int e = 0; e < 4; ++e)
-                                if (mt + c0 + e0 + e < M)
-                                    y[int64_t(mt + c0 + e0 + e) * N + n] =
-                                        __fadd_rn(old[e], __uint_as_float(v[e0 + e]));
-                        }
-                    } else if (n < N) {
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            const int m = mt + c0 + e;
-                            if (m < M) epi_store(epi, Y, m, n, N, __uint_as_float(v[e]));
-                        }
+                        for (int e = 0; e < 16; ++e) part[(c0 + e) * kBN + row] = __uint_as_float(v[e]);
                     }
-                } else {
-                    // token-major partial tile part[m][row] (a warp writes 32 consecutive rows)
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) part[(c0 + e) * kBN + row] = __uint_as_float(v[e]);
                 }
+                // the accumulator may be overwritten by the next item's MMAs
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(acc_empty);
             }
         }
     }
+    // the split-K exchange below (never persistent: one item per CTA) sums that item's tile
+    const Item I_one = item_at(first_item);
+    const int n0 = I_one.n0, m0 = I_one.m0, N = I_one.N, g = I_one.g;
 
     __syncwarp();  // the producer / MMA warps reconverge before the block-wide barriers
     ptx::tc_fence_before();
@@ -602,7 +682,7 @@ template <int FMT, bool SPLIT>
 int smem_bytes(int T, int S, int P) {
     const int need = 1024 + S * P * T * 128 +
                      kRawStages * (RawTraits<FMT>::bytes + RawTraits<FMT>::hbytes + kScaleTile) +
-                     (2 * kRawStages + 3 * S + 1) * 8 + 16;
+                     (2 * kRawStages + 3 * S + 2) * 8 + 16;
     return need > kOneCtaPerSm ? need : kOneCtaPerSm;
 }
 
@@ -793,6 +873,22 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
             }
         }
     }
+    // More items (weight tile x token tile) than SMs with one tile per CTA and no K split:
+    // persistent CTAs, one per SM, each looping over items (barriers, TMEM and the first
+    // copies' latency paid once per CTA; the next item's copies overlap this one's epilogue).
+    int grid_y = tiles, persist = 0;
+    {
+        const int sms = sm_count();
+        const int64_t items = int64_t(grid_x) * tiles;
+        if (P == 1 && splits == 1 && sms > 0 && items > sms && items < (int64_t(1) << 30)) {
+            persist = 1;
+            p.n_tt = grid_x;
+            p.n_items = int32_t(items);
+            grid_x = sms;
+            grid_y = 1;
+        }
+    }
+    p.persist = persist;
     if (!encode_2d(&p.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.X, uint64_t(g.K), uint64_t(g.M),
                    uint64_t(g.K) * 2, kKC, uint32_t(T), CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B))
@@ -831,16 +927,16 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.tmem_cols = kTmemCols;
     p.status = status;
     if (g.fmt == EMB_Q8_0)
-        return split    ? launch_kernel<EMB_Q8_0, true, 1>(p, grid_x, tiles, pdl, s)
-               : P == 2 ? launch_kernel<EMB_Q8_0, false, 2>(p, grid_x, tiles, pdl, s)
-                        : launch_kernel<EMB_Q8_0, false, 1>(p, grid_x, tiles, pdl, s);
+        return split    ? launch_kernel<EMB_Q8_0, true, 1>(p, grid_x, grid_y, pdl, s)
+               : P == 2 ? launch_kernel<EMB_Q8_0, false, 2>(p, grid_x, grid_y, pdl, s)
+                        : launch_kernel<EMB_Q8_0, false, 1>(p, grid_x, grid_y, pdl, s);
     if (g.fmt == EMB_Q4_0)
-        return split    ? launch_kernel<EMB_Q4_0, true, 1>(p, grid_x, tiles, pdl, s)
-               : P == 2 ? launch_kernel<EMB_Q4_0, false, 2>(p, grid_x, tiles, pdl, s)
-                        : launch_kernel<EMB_Q4_0, false, 1>(p, grid_x, tiles, pdl, s);
-    return split    ? launch_kernel<EMB_Q6_0, true, 1>(p, grid_x, tiles, pdl, s)
-           : P == 2 ? launch_kernel<EMB_Q6_0, false, 2>(p, grid_x, tiles, pdl, s)
-                    : launch_kernel<EMB_Q6_0, false, 1>(p, grid_x, tiles, pdl, s);
+        return split    ? launch_kernel<EMB_Q4_0, true, 1>(p, grid_x, grid_y, pdl, s)
+               : P == 2 ? launch_kernel<EMB_Q4_0, false, 2>(p, grid_x, grid_y, pdl, s)
+                        : launch_kernel<EMB_Q4_0, false, 1>(p, grid_x, grid_y, pdl, s);
+    return split    ? launch_kernel<EMB_Q6_0, true, 1>(p, grid_x, grid_y, pdl, s)
+           : P == 2 ? launch_kernel<EMB_Q6_0, false, 2>(p, grid_x, grid_y, pdl, s)
+                    : launch_kernel<EMB_Q6_0, false, 1>(p, grid_x, grid_y, pdl, s);
 }
 
 }  // namespace emb
