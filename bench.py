@@ -661,9 +661,10 @@ def kernel_traffic(workload, w):
     try:
         with open(path) as fh:
             d = json.load(fh)
-        with open(os.path.join(ROOT, d["source"]), "rb") as fh:
-            if hashlib.sha256(fh.read()).hexdigest() != d["source_sha256"]:
-                return None   # the kernel changed since the counters were taken
+        for src in d["sources"]:
+            with open(os.path.join(ROOT, src["path"]), "rb") as fh:
+                if hashlib.sha256(fh.read()).hexdigest() != src["sha256"]:
+                    return None   # the kernels changed since the counters were taken
         return d.get(wl.FMT_NAMES[w.fmt])
     except (OSError, ValueError, KeyError):
         return None
