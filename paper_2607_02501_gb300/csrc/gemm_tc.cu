@@ -63,6 +63,7 @@ constexpr int kMaxStages = 8;              // A/X ring depth, at most
 
 struct GemmParams {
     CUtensorMap x_map;                     // X [M][K] bf16, box {64, T}, 128B swizzle
+    const __nv_bfloat16* X;                // the same X (for its L2 prefetch)
     CUtensorMap codes_map[kMaxGroup];      // codes [N][row bytes] u8, box {128, 128}, 128B swizzle
     CUtensorMap scales_map[kMaxGroup];     // scales [N][ldS] u16, box {8, 128}
     CUtensorMap high_map[kMaxGroup];       // Q6_0 high bits [N][K/4] u8, box {64, 128}, no swizzle
@@ -275,8 +276,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 };
                 if (!waited) {
                     // the first raw stages before griddepcontrol.wait: weights never depend on
-                    // the previous launch; X may be written by it
+                    // the previous launch; X may be written by it, so only its rows' way towards
+                    // L2 starts now (a hint: the TMA loads after the wait read the written values)
                     for (; raw_issued < nr && raw_issued < kRawStages; ++raw_issued) issue_raw(raw_issued);
+                    const int x_rows = min(M - I.m0, P * T);
+                    if (x_rows > 0 && I.n0 == 0 && I.g == 0 && split == 0)  // one CTA per token tile
+                        ptx::prefetch_l2(reinterpret_cast<const uint8_t*>(p.X) + int64_t(I.m0) * K * 2,
+                                         uint32_t(min(int64_t(x_rows) * K * 2, int64_t(1) << 20)));
                     ptx::griddep_wait();
                     waited = true;
                 }
@@ -919,6 +925,7 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.n_mats = g.n_mats;
     p.M = int32_t(g.M);
     p.K = int32_t(g.K);
+    p.X = g.X;
     p.T = T;
     p.P = P;
     p.stages = S;

@@ -102,6 +102,11 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const __grid_constant__ GemvPa
     const int U = p.U;
 
     griddep_launch_dependents();
+    // the activation rows towards L2 while the previous launch finishes (measured on GB300:
+    // cold, they arrive ~2 us after the dependency wait, behind the weight stream); one CTA
+    // per row block asks, since every CTA reads the same rows
+    if (t == 0 && blockIdx.x == 0)
+        ptx::prefetch_l2(p.X + int64_t(m0) * p.K, uint32_t(min(MT, p.M - m0)) * uint32_t(p.K) * 2u);
 
     uint4 c[R];
     uint2 h[R];  // Q6_0 high bits (unused otherwise)
@@ -351,6 +356,10 @@ __global__ void __launch_bounds__(kStageThreads) gemv_staged_kernel(const __grid
         if constexpr (FMT == EMB_Q6_0)
             ptx::bulk_load(high_s, p.high[g] + int64_t(row0) * high_bytes, hi_bytes, bar_w);
         ptx::bulk_load(scales_b, p.scales[g] + int64_t(row0) * p.ldS, scales_bytes, bar_w);
+        // the activation rows towards L2 while the previous launch finishes (measured on
+        // GB300: cold, they land ~2 us after the dependency wait, behind the weight stream);
+        // one CTA per row block asks, since every CTA reads the same rows
+        if (blockIdx.x == 0) ptx::prefetch_l2(p.X + int64_t(m0) * p.K, uint32_t(mt) * uint32_t(p.K) * 2u);
     }
     ptx::griddep_launch_dependents();
     // weights do not depend on earlier launches; X and Y may
@@ -687,6 +696,7 @@ __global__ void __launch_bounds__(kMmaThreads) gemv_q4_mma_kernel(const __grid_c
             ptx::bulk_load(codes_s + r * p.pitch, src_c + int64_t(r) * row_bytes, uint32_t(row_bytes), bar_w);
             ptx::bulk_load(scales_s + r * p.spitch, src_s + int64_t(r) * p.ldS, uint32_t(p.ldS * 2), bar_w);
         }
+        if (lane == 0 && blockIdx.x == 0) ptx::prefetch_l2(p.X, uint32_t(p.M) * uint32_t(p.K) * 2u);  // towards L2
     }
     ptx::griddep_launch_dependents();
     // weights do not depend on earlier launches; X and Y may

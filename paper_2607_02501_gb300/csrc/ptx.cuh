@@ -106,6 +106,13 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
         "l"(src), "r"(bytes), "r"(smem_u32(bar))
         : "memory");
 }
+// Bring `bytes` (a multiple of 16, 16-byte aligned) of global memory towards L2 without
+// waiting. A hint only: it returns no data, so it may run before the data's producer has
+// finished (L2 is the point of coherence; the real load after the dependency wait reads the
+// producer's values).
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(tmap) : "memory");
 }
