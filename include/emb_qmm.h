@@ -183,10 +183,13 @@ typedef struct {
 
 /* Section 3.2, principle 2 (buffer reuse: the caller owns every buffer of a chain,
  * the library allocates nothing).
- * Bytes of device workspace emb_qlayer_seq needs for these layers at this M. This build's
- * kernels need none: the answer is 0 for every valid chain (so EMB_ENOSPC does not occur
- * and the workspace arguments of emb_qlayer_seq / emb_chain_create are reserved).
- * Returns (size_t)-1 for invalid arguments. */
+ * Bytes of device workspace with which emb_qlayer_seq / emb_chain_create run these layers
+ * at this M on the current device with their fastest schedule. 0 when no launch of the
+ * chain wants one (every M <= 4 chain; prefill layers whose tiles already fill the SMs).
+ * Otherwise some tensor-core launch (M >= 128) would split the k range of its tiles evenly
+ * over all SMs ("stream-K") and add the partial tiles through the workspace: 4 KB of
+ * flags, then one fp32 partial tile per SM, a few MB to about 35 MB in all. The answer
+ * depends on the device's SM count. Returns (size_t)-1 for invalid arguments. */
 EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M);
 
 /* Run n_layers linears in order on `stream`, all with M tokens (the paper's
@@ -201,8 +204,15 @@ EMB_API size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, 
  * turn. A layer's W_blocks may not overlap the Y of the same or an earlier
  * layer, and its X may not overlap its own Y (EMB_EINVAL); an unknown epilogue,
  * or a gated one with odd N, is EMB_EINVAL. The call enqueues kernels only, so it may
- * be captured into a CUDA graph and replayed. workspace / ws_bytes: reserved; this
- * build reads neither (emb_qlayer_seq_workspace() is 0), NULL / 0 are fine. */
+ * be captured into a CUDA graph and replayed.
+ * workspace / ws_bytes: NULL, or device memory of at least emb_qlayer_seq_workspace()
+ * bytes (EMB_ENOSPC if smaller), 256-byte aligned (EMB_EALIGN), zero-filled before its
+ * first use. A call leaves it ready for the next one (its first 4 KB, the flags, back at
+ * zero) unless it reports EMB_ETIMEOUT: then zero it again before reusing it. With NULL
+ * the launches take schedules that need none. The
+ * results are deterministic either way, but the two schedules add the k range in different
+ * pieces, so they agree within the accuracy bound, not bitwise. One workspace serves one
+ * stream at a time: calls that may run concurrently need separate workspaces. */
 EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M,
                           void* workspace, size_t ws_bytes, emb_stream_t stream);
 
@@ -213,7 +223,8 @@ EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_
  * every later launch of a call does. Precondition: the weights of the call are not
  * written by the launch enqueued on `stream` just before the call (weights produced
  * further back, e.g. by emb_quantize_* followed by any other launch or a synchronisation,
- * are fine). Results are bitwise those of emb_qlayer_seq. Errors as emb_qlayer_seq. */
+ * are fine). No workspace: results are bitwise those of emb_qlayer_seq with a NULL
+ * workspace. Errors as emb_qlayer_seq. */
 EMB_API emb_status emb_qlayer_seq_chained(const emb_qlayer* layers, int n_layers, int64_t M,
                                           emb_stream_t stream);
 

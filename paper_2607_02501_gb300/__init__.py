@@ -198,6 +198,16 @@ def emb_qlayer_seq_workspace(layers, M: int) -> int:
     return n
 
 
+def chain_workspace(layers, M: int, device=None):
+    """A zero-filled device buffer of emb_qlayer_seq_workspace(layers, M) bytes on the
+    current (or given) CUDA device, or None when the chain needs none."""
+    import torch
+    n = emb_qlayer_seq_workspace(layers, M)
+    if n == 0:
+        return None
+    return torch.zeros(n, dtype=torch.uint8, device=device if device is not None else "cuda")
+
+
 def emb_qlayer_seq(layers, M: int, workspace=None, ws_bytes: int = 0, stream=None) -> None:
     arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
     _check(lib().emb_qlayer_seq(arr, len(arr), M, _ptr(workspace), ws_bytes, _stream(stream)),
@@ -233,11 +243,14 @@ class RecordedChain:
     """emb_qlayer_seq recorded once (emb_chain_create) and replayed with one call per
     step. Holds the specs so that every buffer the recording points at stays alive."""
 
-    def __init__(self, specs, M: int):
+    def __init__(self, specs, M: int, workspace: bool = True):
         self.specs = list(specs)
         self.layers = make_layers(self.specs)
         self.M = M
-        self.handle = emb_chain_create(self.layers, M)
+        # the workspace the chain's fastest schedule wants (zero-filled; None if none)
+        self.workspace = chain_workspace(self.layers, M) if workspace else None
+        ws = self.workspace
+        self.handle = emb_chain_create(self.layers, M, ws, 0 if ws is None else ws.numel())
 
     def launch(self, stream=None) -> None:
         emb_chain_launch(self.handle, stream)

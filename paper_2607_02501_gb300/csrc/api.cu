@@ -272,7 +272,28 @@ static emb_status prepare_seq(const emb_qlayer* layers, int n_layers, int64_t M,
 
 size_t emb_qlayer_seq_workspace(const emb_qlayer* layers, int n_layers, int64_t M) {
     if (check_seq(layers, n_layers, M) != EMB_OK) return size_t(-1);
-    return 0;
+    std::vector<GroupRef> refs;
+    if (prepare_seq(layers, n_layers, M, refs) != EMB_OK) return 0;  // unsupported here: the call fails anyway
+    size_t need = 0;
+    if (M > kGemvMaxM)
+        for (const GroupRef& g : refs) need = std::max(need, gemm_tc_workspace(g));
+    return need;
+}
+
+// The workspace of a chain: NULL (schedules that need none), else 256-byte aligned and at
+// least emb_qlayer_seq_workspace() bytes; every group of the chain uses it in turn.
+static emb_status attach_workspace(std::vector<GroupRef>& refs, int64_t M, void* workspace, size_t ws_bytes) {
+    if (!workspace) return EMB_OK;
+    if (!aligned(workspace, 256)) return EMB_EALIGN;
+    size_t need = 0;
+    if (M > kGemvMaxM)
+        for (const GroupRef& g : refs) need = std::max(need, gemm_tc_workspace(g));
+    if (ws_bytes < need) return EMB_ENOSPC;
+    for (GroupRef& g : refs) {
+        g.ws = workspace;
+        g.ws_bytes = ws_bytes;
+    }
+    return EMB_OK;
 }
 
 static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s, bool first_pdl) {
@@ -288,10 +309,10 @@ static emb_status enqueue_seq(const std::vector<GroupRef>& refs, cudaStream_t s,
 
 emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
                           size_t ws_bytes, emb_stream_t stream) {
-    (void)workspace;  // reserved: this build's kernels need no workspace
-    (void)ws_bytes;
     std::vector<GroupRef> refs;
-    const emb_status st = prepare_seq(layers, n_layers, M, refs);
+    emb_status st = prepare_seq(layers, n_layers, M, refs);
+    if (st != EMB_OK) return st;
+    st = attach_workspace(refs, M, workspace, ws_bytes);
     if (st != EMB_OK) return st;
     return enqueue_seq(refs, reinterpret_cast<cudaStream_t>(stream), false);
 }
@@ -315,12 +336,12 @@ extern "C" {
 
 emb_status emb_chain_create(const emb_qlayer* layers, int n_layers, int64_t M, void* workspace,
                             size_t ws_bytes, emb_chain_t* chain) {
-    (void)workspace;  // reserved, as for emb_qlayer_seq
-    (void)ws_bytes;
     if (!chain) return EMB_EINVAL;
     *chain = nullptr;
     std::vector<GroupRef> refs;
     emb_status st = prepare_seq(layers, n_layers, M, refs);
+    if (st != EMB_OK) return st;
+    st = attach_workspace(refs, M, workspace, ws_bytes);
     if (st != EMB_OK) return st;
     // capture the chain's launches on a private stream (thread-local capture mode, so other
     // threads' CUDA calls are unaffected), then instantiate the graph once

@@ -127,6 +127,8 @@ struct GroupRef {
     int64_t M;
     int64_t K;
     int64_t ldS;
+    void* ws;               // caller workspace for the tensor-core GEMM's stream-K schedule, or NULL
+    size_t ws_bytes;
 };
 
 // Weight-streaming GEMV for small M (register dequant, shuffle reductions).
@@ -137,6 +139,9 @@ cudaError_t launch_gemv(const GroupRef& g, bool pdl, int* status, cudaStream_t s
 // Tensor-core GEMM (tcgen05 + TMEM) for larger M.
 cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s);
 bool gemm_tc_supported(const GroupRef& g);
+// Bytes of zero-filled workspace the GEMM's stream-K schedule wants for this group on the
+// current device (0: the group's plan needs none).
+size_t gemm_tc_workspace(const GroupRef& g);
 
 // Layer steps around the linears (csrc/layer_ops.cu): RMSNorm of the fp32 residual into
 // bf16, rotary embedding in place, grouped-head attention over a prefix cache and the

@@ -82,6 +82,10 @@ struct GemmParams {
     uint32_t tmem_cols;
     int32_t persist;                       // 1: CTAs loop over items (no K split)
     int32_t n_tt, n_items;                 // persistent: token tiles per weight tile, items
+    int32_t streamk;                       // 1: the items' raw stages split evenly over the CTAs
+    int32_t slot_floats;                   // stream-K: floats of one partial tile (P * T * 128)
+    float* ws_part;                        // stream-K: one partial-tile slot per CTA
+    uint32_t* ws_flag;                     // stream-K: one ready flag per CTA (zero between launches)
     int* status;
 };
 
@@ -153,10 +157,11 @@ __device__ __forceinline__ uint32_t a_stage_col(int s, int gap0, int per_gap) {
     return uint32_t(s < per_gap ? gap0 + s * kACols : kAccCols + gap0 + (s - per_gap) * kACols);
 }
 
-template <int FMT, bool SPLIT, int P>
+template <int FMT, bool SPLIT, int P, bool SK>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmParams p) {
     using RT = RawTraits<FMT>;
     static_assert(P == 1 || (P == 2 && !SPLIT), "two token tiles only without the split operand");
+    static_assert(!(SK && SPLIT), "stream-K only without the split operand");
     extern __shared__ uint8_t smem_dyn[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_dyn) + 1023) &
                                                ~uintptr_t(1023));
@@ -173,38 +178,83 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint64_t* ax_empty = a_full + S;
     uint64_t* acc_full = ax_empty + S;
     uint64_t* acc_empty = acc_full + 1;  // the epilogue warps have read the accumulator
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 1);
+    uint64_t* sk_full = acc_empty + 1;   // stream-K head: a chunk of a tail is in the X ring
+    uint64_t* sk_free = sk_full + 1;     // stream-K head: every epilogue warp has added it
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sk_free + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     volatile int* mma_stop = abort_flag + 1;  // set by the waiter warp when a wait gave up
+    int* sk_cnt = const_cast<int*>(mma_stop) + 1;  // stream-K: epilogue warps done with the tail
+    int* sk_seen = sk_cnt + 1;                     // stream-K: epilogue warps done with the head
     // split-K partial tile [T][128] fp32 (token-major): reuses the X ring once every MMA
     // has completed
     float* part = reinterpret_cast<float*>(x_ring);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int M = p.M, K = p.K;
-    // this CTA's K range: split-K over raw stages of 256 (the same for all of its items)
     const int splits = gridDim.z, split = blockIdx.z;
     const int nr_all = (K + kKR - 1) / kKR, nk_all = (K + kKC - 1) / kKC;
-    const int rs0 = split * nr_all / splits, rs1 = (split + 1) * nr_all / splits;
-    const int nr = rs1 - rs0;
-    const int ks0 = rs0 * kStepsPerRaw;
-    const int nk = min(rs1 * kStepsPerRaw, nk_all) - ks0;
-    // Work items (weight tile, token tile). Without p.persist each CTA has one: grid x =
-    // token tile, y = weight tile, z = K split. With p.persist (no K split) CTA c takes items
-    // c, c + gridDim.x, ... in the order of token tiles within weight tiles, so the CTAs at
-    // work on a weight tile at one time read it once from HBM and then from L2. Rings and
-    // barrier phases run on across items; the next item's codes and activations stream in
-    // while the current item's epilogue drains the accumulator.
+    // Work items (weight tile, token tile), each over a range of raw stages (256 k) of its
+    // row. Three schedules:
+    //  * one item per CTA: grid x = token tile, y = weight tile, z = K split (a cluster
+    //    along z shares one item; split s takes raw stages [s*nr/splits, (s+1)*nr/splits));
+    //  * p.persist: CTA c takes whole items c, c + gridDim.x, ... in the order of token
+    //    tiles within weight tiles, so the CTAs at work on a weight tile at one time read it
+    //    once from HBM and then from L2;
+    //  * SK (stream-K): the raw stages of all items, item after item, are cut into gridDim.x
+    //    equal ranges, one per CTA, so every SM gets the same work whatever the tile count.
+    //    A range starts inside an item (a "tail": its sum is left in the CTA's workspace
+    //    slot, flagged ready) and/or ends inside one (a "head" holding k = 0: its CTA adds
+    //    the tails of the CTAs after it, in CTA order, i.e. in k order, and runs the
+    //    epilogue). Results are deterministic for a given grid.
+    // With more than one item, rings and barrier phases run on across items; the next
+    // item's codes and activations stream in while the current one's epilogue drains the
+    // accumulator.
     const bool persist = p.persist != 0;
-    const int first_item = persist ? int(blockIdx.x) : 0;
-    const int item_stride = persist ? int(gridDim.x) : 1;
-    const int n_items = persist ? p.n_items : 1;
+    constexpr bool streamk = SK;  // a separate instance: the plain schedules carry none of its code
+    const int64_t sk_units = int64_t(p.n_items) * nr_all;  // stream-K: raw stages of all items
+    // this CTA's segments j = 0 .. n_seg-1: item it0 + j*it_stride over raw stages [r0, r1),
+    // r0 = 0 but for the first, r1 = nr_all but for the last
+    int it0 = 0, it_stride = 1, r0_first = 0, r1_last = nr_all, n_seg = 1;
+    if (streamk) {
+        const int64_t u_beg = int64_t(blockIdx.x) * sk_units / gridDim.x;
+        const int64_t u_end = int64_t(blockIdx.x + 1) * sk_units / gridDim.x;
+        const int64_t last = (u_end - 1) / nr_all;
+        it0 = int(u_beg / nr_all);
+        r0_first = int(u_beg - int64_t(it0) * nr_all);
+        r1_last = int(u_end - last * nr_all);
+        n_seg = u_end > u_beg ? int(last) - it0 + 1 : 0;
+    } else if (persist) {
+        it0 = int(blockIdx.x);
+        it_stride = int(gridDim.x);
+        n_seg = int(blockIdx.x) < p.n_items ? (p.n_items - int(blockIdx.x) + int(gridDim.x) - 1) / int(gridDim.x) : 0;
+    } else {
+        r0_first = split * nr_all / splits;
+        r1_last = (split + 1) * nr_all / splits;
+    }
+    // stream-K: a head (last segment holding k = 0 of an item that goes on) adds the tails of
+    // CTAs [blockIdx.x + 1, sk_q_end): those whose ranges start inside that item
+    int sk_q_end = int(blockIdx.x) + 1;
+    if (streamk && n_seg > 0 && r1_last < nr_all && (n_seg > 1 || r0_first == 0)) {
+        const int64_t item_end = int64_t(it0 + n_seg) * nr_all;
+        while (sk_q_end < int(gridDim.x) && int64_t(sk_q_end) * sk_units / gridDim.x < item_end) ++sk_q_end;
+    }
+    struct Seg {
+        int it, r0, r1;  // item, raw stages [r0, r1) of its row
+    };
+    auto seg_at = [&](int j) {
+        Seg s;
+        s.it = it0 + j * it_stride;
+        s.r0 = j == 0 ? r0_first : 0;
+        s.r1 = j == n_seg - 1 ? r1_last : nr_all;
+        return s;
+    };
+    auto seg_nk = [&](const Seg& s) { return min(s.r1 * kStepsPerRaw, nk_all) - s.r0 * kStepsPerRaw; };
     struct Item {
         int g, n0, m0, N;
     };
     auto item_at = [&](int it) {
-        const int tt = persist ? it % p.n_tt : int(blockIdx.x);
-        const int tile = persist ? it / p.n_tt : int(blockIdx.y);
+        const int tt = (persist || streamk) ? it % p.n_tt : int(blockIdx.x);
+        const int tile = (persist || streamk) ? it / p.n_tt : int(blockIdx.y);
         Item r;
         r.g = 0;
 #pragma unroll
@@ -228,8 +278,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         ptx::mbar_init(acc_full, 1);
         ptx::mbar_init(acc_empty, kDeqWarps);
+        ptx::mbar_init(sk_full, 1);
+        ptx::mbar_init(sk_free, kDeqWarps);
         *abort_flag = 0;
         *mma_stop = 0;
+        *sk_cnt = 0;
+        *sk_seen = 0;
         ptx::fence_mbar_init();
         ptx::prefetch_tmap(&p.x_map);
         for (int i = 0; i < p.n_mats; ++i) {
@@ -256,13 +310,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint64_t pol_x = ptx::policy_evict_last();
             int raw_issued = 0, x_issued = 0;  // over all items of the CTA
             bool stop = false, waited = false;
-            for (int it = first_item; it < n_items && !stop; it += item_stride, ++items_done) {
-                const Item I = item_at(it);
-                const int rbase = items_done * nr, xbase = items_done * nk;
-                auto issue_raw = [&](int r) {  // raw stage r of this item (global rbase + r)
+            int rbase = 0, xbase = 0;  // raw stages and steps of the earlier segments
+            for (int j = 0; j < n_seg && !stop; ++j, ++items_done) {
+                const Seg sg = seg_at(j);
+                const Item I = item_at(sg.it);
+                const int nr = sg.r1 - sg.r0, nk = seg_nk(sg), ks0 = sg.r0 * kStepsPerRaw;
+                auto issue_raw = [&](int r) {  // raw stage r of this segment (global rbase + r)
                     const int rg_all = rbase + r;
                     const int slot = rg_all % kRawStages;
-                    const int rg = rs0 + r;  // raw stage index within the whole row
+                    const int rg = sg.r0 + r;  // raw stage index within the whole row
                     ptx::mbar_arrive_expect_tx(&raw_full[slot], RT::bytes + RT::hbytes + kScaleTile);
 #pragma unroll
                     for (int pl = 0; pl < RT::planes; ++pl)
@@ -280,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     // L2 starts now (a hint: the TMA loads after the wait read the written values)
                     for (; raw_issued < nr && raw_issued < kRawStages; ++raw_issued) issue_raw(raw_issued);
                     const int x_rows = min(M - I.m0, P * T);
-                    if (x_rows > 0 && I.n0 == 0 && I.g == 0 && split == 0)  // one CTA per token tile
+                    if (x_rows > 0 && I.n0 == 0 && I.g == 0 && sg.r0 == 0)  // one CTA per token tile
                         ptx::prefetch_l2(reinterpret_cast<const uint8_t*>(p.X) + int64_t(I.m0) * K * 2,
                                          uint32_t(min(int64_t(x_rows) * K * 2, int64_t(1) << 20)));
                     ptx::griddep_wait();
@@ -314,6 +370,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                                          (ks0 + i) * kKC, I.m0 + q * T, pol_x);
                     ++x_issued;
                 }
+                rbase += nr;
+                xbase += nk;
             }
             // every issued copy must land before this CTA's shared memory can be released
             for (int r = raw_issued - 1; r >= 0 && r >= raw_issued - kRawStages; --r)
@@ -329,9 +387,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         const uint32_t idesc = ptx::idesc_bf16_f32(kBN, T);
         const uint32_t x0 = ptx::smem_u32(x_ring);
         bool stop = false;
-        int commits = 0;  // accumulator commits (one per finished item)
-        for (int it = first_item; it < n_items && !stop; it += item_stride, ++items_done) {
-            const int xbase = items_done * nk;
+        int commits = 0;  // accumulator commits (one per finished segment)
+        int xbase = 0;
+        for (int j = 0; j < n_seg && !stop; ++j, ++items_done) {
+            const int nk = seg_nk(seg_at(j));
             for (int i = 0; i < nk; ++i) {
                 named_sync(1, 64);
                 if (*mma_stop) {
@@ -362,6 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             if (stop) break;
             if (lane == 0) ptx::mma_commit(acc_full);
             ++commits;
+            xbase += nk;
             __syncwarp();
         }
         if (lane == 0 && commits > 0)  // the last item's MMAs finish before TMEM is freed
@@ -374,8 +434,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         // X tile and A tile (and, at an item's first step, for the previous item's epilogue
         // to have read the accumulator) and then releases the MMA warp through named barrier 1.
         bool stop = false;
-        for (int it = first_item; it < n_items && !stop; it += item_stride, ++items_done) {
-            const int xbase = items_done * nk;
+        int xbase = 0;
+        for (int j = 0; j < n_seg && !stop; ++j, ++items_done) {
+            const int nk = seg_nk(seg_at(j));
             for (int i = 0; i < nk; ++i) {
                 const int xs = xbase + i;
                 const int s = xs % S;
@@ -395,6 +456,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     break;
                 }
             }
+            xbase += nk;
         }
     } else if (warp < 2 + kDeqWarps) {
         // ---------------------------------------------------------------- dequant
@@ -405,9 +467,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         const uint32_t a_lane = tmem + (uint32_t(32 * (warp & 3)) << 16) + uint32_t(16 * h);
         const unsigned full = 0xffffffffu;
         bool ok = true;
-        for (int it = first_item; it < n_items && ok; it += item_stride, ++items_done) {
-            const Item I = item_at(it);
-            const int rbase = items_done * nr, xbase = items_done * nk;
+        int rbase = 0, xbase = 0;  // raw stages and steps of the earlier segments
+        for (int j = 0; j < n_seg && ok; ++j, ++items_done) {
+            const Seg sg = seg_at(j);
+            const Item I = item_at(sg.it);
+            const int nr = sg.r1 - sg.r0, nk = seg_nk(sg);
             // Software pipeline: step i's TMEM stores are completed (tcgen05.wait::st) and
             // signalled only after step i+1 has been computed, so the store latency overlaps
             // the next step's arithmetic instead of stalling this warp every step.
@@ -522,6 +586,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             ptx::griddep_wait();  // Y may be read or written by the previous launch
             ok = __all_sync(full, ok && ptx::mbar_wait(acc_full, items_done & 1, abort_flag, p.status,
                                                        kWaitLimitNs));
+            // stream-K: a tail goes to this CTA's workspace slot; a head first adds the tails of
+            // the CTAs after it (those whose ranges start inside this item), in CTA order
+            const bool sk_tail = streamk && sg.r0 > 0;
+            const bool sk_head = streamk && sg.r0 == 0 && sg.r1 < nr_all;
             if (ok) {
                 ptx::tc_fence_after();
                 // warps 2..9: TMEM lane quarter = warp % 4; the two warps of a quarter split the
@@ -537,10 +605,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 const int mt = I.m0 + tt * T;  // first token of that tile
                 void* Y = p.Y[I.g];
                 const int epi = p.epi;
-                for (int c0 = cbeg; c0 < cend; c0 += 16) {
-                    uint32_t v[16];
-                    ptx::tmem_ld_16(taddr + uint32_t(c0), v);
-                    ptx::tmem_ld_wait();
+                // Emit 16 accumulator columns c0 .. c0+15 of this warp's rows, plus (stream-K
+                // head) the staged last tail
+                const uint32_t staged = ptx::smem_u32(x_ring);  // staged tail: [cols][128] fp32
+                bool add_staged = false;
+                auto emit = [&](uint32_t (&v)[16], int c0) {
+                    if (add_staged) {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            v[e] = __float_as_uint(__fadd_rn(
+                                __uint_as_float(v[e]), ptx::ld_shared_f32(staged + uint32_t(((tt * T + c0 + e) * kBN + row) * 4))));
+                    }
                     if (splits == 1) {
                         if (epi >= EMB_EPI_GEGLU) {
                             // gate row n (even lane) and up row n + 1 (the next lane): rows past N
@@ -580,16 +655,103 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 #pragma unroll
                         for (int e = 0; e < 16; ++e) part[(c0 + e) * kBN + row] = __uint_as_float(v[e]);
                     }
+                };
+                if (sk_head) {
+                    // Workspace slots are token-major [P*T][128] fp32. Each tail is staged into the
+                    // (now idle) X ring by bulk copies, in column chunks that fit it. Every tail but
+                    // the last is added into the accumulator in TMEM; the last one, when it fits in
+                    // one chunk, is added by the store pass below.
+                    const int slot_cols = P * T;
+                    const int chunk_cols = min(slot_cols, ((S * P * T) / 4) & ~15);  // X ring bytes / 512
+                    int chunk_no = 0;
+                    for (int q = int(blockIdx.x) + 1; q < sk_q_end && ok; ++q) {
+                        for (int k0 = 0; k0 < slot_cols && ok; k0 += chunk_cols, ++chunk_no) {
+                            const int k1 = min(slot_cols, k0 + chunk_cols);
+                            if (warp == 2 && lane == 0) {
+                                bool good = true;
+                                if (k0 == 0) {
+                                    good = ptx::flag_wait(p.ws_flag + q, abort_flag, p.status, kWaitLimitNs);
+                                    ptx::fence_proxy_async_global();  // the tail's stores, seen by the copy
+                                }
+                                if (good && chunk_no > 0)  // every warp has read the previous chunk
+                                    good = ptx::mbar_wait(sk_free, (chunk_no - 1) & 1, abort_flag, p.status,
+                                                          kWaitLimitNs);
+                                if (good) {
+                                    const uint32_t bytes = uint32_t(k1 - k0) * uint32_t(kBN) * 4u;
+                                    ptx::mbar_arrive_expect_tx(sk_full, bytes);
+                                    ptx::bulk_load(x_ring, p.ws_part + int64_t(q) * p.slot_floats + int64_t(k0) * kBN,
+                                                   bytes, sk_full);
+                                }
+                            }
+                            ok = __all_sync(full, ptx::mbar_wait(sk_full, chunk_no & 1, abort_flag, p.status,
+                                                                 kWaitLimitNs));
+                            if (!ok) break;
+                            if (q == sk_q_end - 1 && chunk_cols == slot_cols) {
+                                add_staged = true;  // the store pass adds it
+                                break;
+                            }
+                            for (int c0 = cbeg; c0 < cend; c0 += 16) {
+                                const int sc = tt * T + c0;  // slot column (chunks are whole 16-column groups)
+                                if (sc < k0 || sc >= k1) continue;
+                                uint32_t v[16];
+                                ptx::tmem_ld_16(taddr + uint32_t(c0), v);
+                                ptx::tmem_ld_wait();
+#pragma unroll
+                                for (int e = 0; e < 16; ++e)
+                                    v[e] = __float_as_uint(__fadd_rn(
+                                        __uint_as_float(v[e]), ptx::ld_shared_f32(staged + uint32_t(((sc - k0 + e) * kBN + row) * 4))));
+                                ptx::tmem_st_16(taddr + uint32_t(c0), v);
+                            }
+                            ptx::tmem_st_wait();
+                            __syncwarp();
+                            if (lane == 0) ptx::mbar_arrive(sk_free);
+                        }
+                    }
+                }
+                if (sk_tail) {
+                    float* slot = p.ws_part + int64_t(blockIdx.x) * p.slot_floats;
+                    for (int c0 = cbeg; c0 < cend; c0 += 16) {
+                        uint32_t v[16];
+                        ptx::tmem_ld_16(taddr + uint32_t(c0), v);
+                        ptx::tmem_ld_wait();
+                        float* dst = slot + int64_t(tt * T + c0) * kBN + row;  // a warp writes 32 consecutive rows
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) __stcg(dst + e * kBN, __uint_as_float(v[e]));
+                    }
+                    // the last of the eight warps to finish publishes the tail
+                    __threadfence();
+                    __syncwarp();
+                    if (lane == 0 && atomicAdd(sk_cnt, 1) == kDeqWarps - 1) {
+                        __threadfence();
+                        ptx::st_release_gpu(p.ws_flag + blockIdx.x, 1u);
+                    }
+                } else if (ok) {
+                    // one TMEM load per wait (two per wait measured slower on GB300: the kernel's
+                    // register count rose by 16 and the main loop lost 10-17 %)
+                    for (int c0 = cbeg; c0 < cend; c0 += 16) {
+                        uint32_t v[16];
+                        ptx::tmem_ld_16(taddr + uint32_t(c0), v);
+                        ptx::tmem_ld_wait();
+                        emit(v, c0);
+                    }
+                }
+                if (sk_head && ok) {
+                    // the last of the eight warps to finish clears the flags it consumed
+                    __syncwarp();
+                    if (lane == 0 && atomicAdd(sk_seen, 1) == kDeqWarps - 1)
+                        for (int q = int(blockIdx.x) + 1; q < sk_q_end; ++q) ptx::st_relaxed_gpu(p.ws_flag + q, 0u);
                 }
                 // the accumulator may be overwritten by the next item's MMAs
                 ptx::tc_fence_before();
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(acc_empty);
             }
+            rbase += nr;
+            xbase += nk;
         }
     }
     // the split-K exchange below (never persistent: one item per CTA) sums that item's tile
-    const Item I_one = item_at(first_item);
+    const Item I_one = item_at(0);
     const int n0 = I_one.n0, m0 = I_one.m0, N = I_one.N, g = I_one.g;
 
     __syncwarp();  // the producer / MMA warps reconverge before the block-wide barriers
@@ -688,7 +850,7 @@ template <int FMT, bool SPLIT>
 int smem_bytes(int T, int S, int P) {
     const int need = 1024 + S * P * T * 128 +
                      kRawStages * (RawTraits<FMT>::bytes + RawTraits<FMT>::hbytes + kScaleTile) +
-                     (2 * kRawStages + 3 * S + 2) * 8 + 16;
+                     (2 * kRawStages + 3 * S + 4) * 8 + 32;
     return need > kOneCtaPerSm ? need : kOneCtaPerSm;
 }
 
@@ -714,7 +876,7 @@ int pick_stages_pair(int T, int& gap0, int& per_gap) {
     return S;
 }
 
-template <int FMT, bool SPLIT, int P>
+template <int FMT, bool SPLIT, int P, bool SK = false>
 cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl, cudaStream_t s) {
     // grid: x = token tile (fastest, so the CTAs sharing a weight tile run together and
     // read it from L2 after the first), y = weight-row tile, z = K split (one cluster)
@@ -728,7 +890,7 @@ cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl,
     {
         std::lock_guard<std::mutex> lock(mu);
         if (dev < 0 || dev >= 64 || !done[dev]) {
-            e = cudaFuncSetAttribute(gemm_tc_kernel<FMT, SPLIT, P>,
+            e = cudaFuncSetAttribute(gemm_tc_kernel<FMT, SPLIT, P, SK>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
             if (e != cudaSuccess) return e;
             if (dev >= 0 && dev < 64) done[dev] = true;
@@ -755,7 +917,7 @@ cudaError_t launch_kernel(const GemmParams& p, int grid_x, int grid_y, bool pdl,
     }
     cfg.attrs = attr;
     cfg.numAttrs = na;
-    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<FMT, SPLIT, P>, p);
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<FMT, SPLIT, P, SK>, p);
 }
 
 int sm_count() {
@@ -798,9 +960,25 @@ bool gemm_tc_supported(const GroupRef& g) {
            (g.fmt != EMB_Q6_0 || g.K % 64 == 0) && encode_fn() != nullptr;
 }
 
-cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s) {
-    GemmParams p;
-    memset(&p, 0, sizeof(p));
+namespace {
+
+struct GemmPlan {
+    int T = 0, S = 0, P = 1, splits = 1;
+    int grid_x = 0, grid_y = 0, persist = 0, streamk = 0;
+    int a_gap0 = 0, a_per_gap = 0, n_tt = 0, n_items = 0;
+    size_t ws_bytes = 0;  // stream-K workspace: flags, then grid_x partial-tile slots
+};
+
+// Stream-K workspace of a plan: one 32-bit flag per CTA in the first kSkFlagBytes, then one
+// partial tile (P * T tokens x 128 rows, fp32) per CTA, each slot 256-byte aligned.
+constexpr int kSkFlagBytes = 4096;  // room for 1024 CTAs
+size_t sk_slot_bytes(int P, int T) { return size_t(roundup(int64_t(P) * T * kBN * 4, 256)); }
+size_t sk_ws_bytes(int G, int P, int T) { return kSkFlagBytes + size_t(G) * sk_slot_bytes(P, T); }
+
+// The launch shape of one group. With streamk_ok the plan may take the stream-K schedule,
+// which needs plan.ws_bytes of zero-filled workspace.
+GemmPlan plan_gemm(const GroupRef& g, bool streamk_ok) {
+    GemmPlan pl;
     int tiles = 0;
     for (int i = 0; i < g.n_mats; ++i) tiles += int((g.mats[i].N + kBN - 1) / kBN);
     // one token tile per CTA: balanced tiles of at most 256, rounded up to the MMA's N granule
@@ -874,8 +1052,8 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
                 S = S2;
                 splits = 1;
                 grid_x = int(t2 / 2);
-                p.a_gap0 = gap0;
-                p.a_per_gap = per_gap;
+                pl.a_gap0 = gap0;
+                pl.a_per_gap = per_gap;
             }
         }
     }
@@ -888,13 +1066,108 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
         const int64_t items = int64_t(grid_x) * tiles;
         if (P == 1 && splits == 1 && sms > 0 && items > sms && items < (int64_t(1) << 30)) {
             persist = 1;
-            p.n_tt = grid_x;
-            p.n_items = int32_t(items);
+            pl.n_tt = grid_x;
+            pl.n_items = int32_t(items);
             grid_x = sms;
             grid_y = 1;
         }
     }
-    p.persist = persist;
+    pl.T = T;
+    pl.S = S;
+    pl.P = P;
+    pl.splits = splits;
+    pl.grid_x = grid_x;
+    pl.grid_y = grid_y;
+    pl.persist = persist;
+    // Stream-K: when the waves of whole items leave SMs idle (a last wave that is mostly
+    // empty), cut the raw stages of all items into one equal range per SM. Both plans are
+    // costed with per 64-k step max(900, 4.1 per token of the CTA) cycles (measured on
+    // GB300: 922 at one tile of 208, 1170 at two of 144) plus ~3900 of fill per CTA (and
+    // ~5000 for a K split's cluster exchange); stream-K adds ~17000 for writing, publishing,
+    // staging and adding a partial tile and ~3300 for every further tail a head adds
+    // (per-CTA %globaltimer stamps: 147 KB written in ~3 us, staged and added in ~1.7 us, a
+    // slower store pass after it). So it is taken only where it is clearly faster (10 %):
+    // Llama-7B gate/up at M = 280, 172 tiles on 152 SMs, 84 -> 61 us; the q/k/v, o and down
+    // projections, whose tiles fill more of the SMs, gain nothing or lose.
+    const int sms = sm_count();
+    if (streamk_ok && !split && g.M >= 128 && sms > 0) {
+        const int64_t nr_all = (g.K + kKR - 1) / kKR;
+        const double nk = double((g.K + kKC - 1) / kKC);
+        auto step = [](int Pc, int Tc) { return std::max(900.0, 4.1 * Pc * Tc); };
+        double cur;
+        if (pl.persist)
+            cur = double((int64_t(pl.n_items) + sms - 1) / sms) * nk * step(P, T) + 3900.0;
+        else
+            cur = double((int64_t(grid_x) * grid_y * splits + sms - 1) / sms) *
+                  (std::ceil(nk / splits) * step(P, T) + 3900.0 + (splits > 1 ? 5000.0 : 0.0));
+        struct Cand { int P, T, S, gap0, per_gap; int64_t n_tt; };
+        Cand cands[2];
+        int nc = 0;
+        {
+            const int64_t tt1 = (g.M + 255) / 256;
+            const int T1 = int(roundup((g.M + tt1 - 1) / tt1, 16));
+            const int S1 = g.fmt == EMB_Q8_0   ? pick_stages<EMB_Q8_0, false>(T1)
+                           : g.fmt == EMB_Q4_0 ? pick_stages<EMB_Q4_0, false>(T1)
+                                               : pick_stages<EMB_Q6_0, false>(T1);
+            cands[nc++] = Cand{1, T1, S1, 0, 0, tt1};
+            const int64_t t2 = 2 * ((g.M + 447) / 448);
+            const int T2 = int(roundup((g.M + t2 - 1) / t2, 16));
+            int gap0 = 0, per_gap = 0;
+            const int S2 = g.fmt == EMB_Q8_0   ? pick_stages_pair<EMB_Q8_0>(T2, gap0, per_gap)
+                           : g.fmt == EMB_Q4_0 ? pick_stages_pair<EMB_Q4_0>(T2, gap0, per_gap)
+                                               : pick_stages_pair<EMB_Q6_0>(T2, gap0, per_gap);
+            if (S2 >= 2 && T2 <= 224) cands[nc++] = Cand{2, T2, S2, gap0, per_gap, t2 / 2};
+        }
+        double best = cur / 1.1;
+        for (int c = 0; c < nc; ++c) {
+            const Cand& cd = cands[c];
+            const int64_t items = cd.n_tt * tiles;
+            const int64_t U = items * nr_all;
+            if (items >= (int64_t(1) << 30) || U >= (int64_t(1) << 31)) continue;
+            const int64_t G = std::min<int64_t>(std::min(sms, kSkFlagBytes / 4), U);
+            // a head adds the tails of the CTAs whose ranges start inside its item
+            const int64_t per = std::max<int64_t>(1, U / G);
+            const double tails = double(std::max<int64_t>(1, (nr_all + per - 1) / per));
+            const double t = double((U + G - 1) / G) * kStepsPerRaw * step(cd.P, cd.T) + 3900.0 + 17000.0 +
+                             3300.0 * (tails - 1.0);
+            if (t < best) {
+                best = t;
+                pl.T = cd.T;
+                pl.S = cd.S;
+                pl.P = cd.P;
+                pl.a_gap0 = cd.gap0;
+                pl.a_per_gap = cd.per_gap;
+                pl.splits = 1;
+                pl.persist = 1;
+                pl.streamk = 1;
+                pl.n_tt = int(cd.n_tt);
+                pl.n_items = int(items);
+                pl.grid_x = int(G);
+                pl.grid_y = 1;
+                pl.ws_bytes = sk_ws_bytes(int(G), cd.P, cd.T);
+            }
+        }
+    }
+    return pl;
+}
+
+cudaError_t launch_plan(const GroupRef& g, const GemmPlan& pl, bool pdl, int* status, cudaStream_t s) {
+    GemmParams p;
+    memset(&p, 0, sizeof(p));
+    const int T = pl.T, S = pl.S, P = pl.P, splits = pl.splits, grid_x = pl.grid_x, grid_y = pl.grid_y;
+    const bool split = g.K < 1024 || g.precise;
+    p.persist = pl.persist;
+    p.streamk = pl.streamk;
+    p.n_tt = pl.n_tt;
+    p.n_items = pl.n_items;
+    p.a_gap0 = pl.a_gap0;
+    p.a_per_gap = pl.a_per_gap;
+    if (pl.streamk) {
+        p.slot_floats = int32_t(sk_slot_bytes(P, T) / 4);
+        p.ws_flag = static_cast<uint32_t*>(g.ws);
+        p.ws_part = reinterpret_cast<float*>(static_cast<uint8_t*>(g.ws) + kSkFlagBytes);
+    }
+    int tiles = 0;
     if (!encode_2d(&p.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, g.X, uint64_t(g.K), uint64_t(g.M),
                    uint64_t(g.K) * 2, kKC, uint32_t(T), CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B))
@@ -933,6 +1206,16 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     p.epi = g.epi;
     p.tmem_cols = kTmemCols;
     p.status = status;
+    if (pl.streamk) {
+        if (g.fmt == EMB_Q8_0)
+            return P == 2 ? launch_kernel<EMB_Q8_0, false, 2, true>(p, grid_x, grid_y, pdl, s)
+                          : launch_kernel<EMB_Q8_0, false, 1, true>(p, grid_x, grid_y, pdl, s);
+        if (g.fmt == EMB_Q4_0)
+            return P == 2 ? launch_kernel<EMB_Q4_0, false, 2, true>(p, grid_x, grid_y, pdl, s)
+                          : launch_kernel<EMB_Q4_0, false, 1, true>(p, grid_x, grid_y, pdl, s);
+        return P == 2 ? launch_kernel<EMB_Q6_0, false, 2, true>(p, grid_x, grid_y, pdl, s)
+                      : launch_kernel<EMB_Q6_0, false, 1, true>(p, grid_x, grid_y, pdl, s);
+    }
     if (g.fmt == EMB_Q8_0)
         return split    ? launch_kernel<EMB_Q8_0, true, 1>(p, grid_x, grid_y, pdl, s)
                : P == 2 ? launch_kernel<EMB_Q8_0, false, 2>(p, grid_x, grid_y, pdl, s)
@@ -944,6 +1227,21 @@ cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_
     return split    ? launch_kernel<EMB_Q6_0, true, 1>(p, grid_x, grid_y, pdl, s)
            : P == 2 ? launch_kernel<EMB_Q6_0, false, 2>(p, grid_x, grid_y, pdl, s)
                     : launch_kernel<EMB_Q6_0, false, 1>(p, grid_x, grid_y, pdl, s);
+}
+
+}  // namespace
+
+size_t gemm_tc_workspace(const GroupRef& g) {
+    if (!gemm_tc_supported(g)) return 0;
+    return plan_gemm(g, true).ws_bytes;
+}
+
+// The stream-K schedule runs only with a caller workspace large enough for it (its size
+// is what gemm_tc_workspace reports); without one the group takes the plan without it.
+cudaError_t launch_gemm_tc(const GroupRef& g, bool pdl, int* status, cudaStream_t s) {
+    GemmPlan pl = plan_gemm(g, g.ws != nullptr);
+    if (pl.streamk && g.ws_bytes < pl.ws_bytes) pl = plan_gemm(g, false);
+    return launch_plan(g, pl, pdl, status, s);
 }
 
 }  // namespace emb

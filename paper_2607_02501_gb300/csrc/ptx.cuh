@@ -70,6 +70,58 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     }
 }
 
+// ------------------------------------------------------------- shared memory
+// Loads through the shared state space (the kernels' shared pointers are generic: they
+// are aligned through integer arithmetic, which hides their space from the compiler).
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t saddr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(saddr));
+    return v;
+}
+__device__ __forceinline__ float ld_shared_f32(uint32_t saddr) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(saddr));
+    return v;
+}
+
+// ------------------------------------------------------------- global flags
+// A 32-bit flag in global memory shared by the CTAs of one grid.
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release_gpu(uint32_t* p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_relaxed_gpu(uint32_t* p, uint32_t v) {
+    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Orders this thread's earlier generic-proxy view of global memory before its later
+// async-proxy (bulk copy) accesses.
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+// Wait until *flag is non-zero (acquire: what its writer published before it is visible).
+// Gives up like mbar_wait.
+__device__ __forceinline__ bool flag_wait(const uint32_t* flag, volatile int* abort, int* status,
+                                          uint64_t limit_ns) {
+    if (ld_acquire_gpu(flag) != 0u) return true;
+    const uint64_t t0 = globaltimer();
+    for (;;) {
+        __nanosleep(64);
+        if (ld_acquire_gpu(flag) != 0u) return true;
+        if (abort != nullptr && *abort) return false;
+        if (globaltimer() - t0 > limit_ns) {
+            if (status) atomicOr(status, kStatusTimeout);
+            if (abort) *abort = 1;
+            return false;
+        }
+    }
+}
+
 // ------------------------------------------------------------------------ TMA
 __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0,
                                             int c1, uint64_t policy) {

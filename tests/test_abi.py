@@ -165,10 +165,22 @@ def test_seq_epilogue_overlap_rules(L):
     assert L.emb_qlayer_seq_workspace(bad, 1, M) == ctypes.c_size_t(-1).value
 
 
-def test_seq_workspace_is_zero_for_valid_chains(L):
+def test_seq_workspace_without_a_device(L):
+    """Decode chains never want a workspace; without a GPU no schedule is planned, so a
+    prefill chain's answer is 0 too (the call itself would fail)."""
     chain = _layers([(0, A, 128, 64, B, C), (1, A + (64 << 20), 256, 64, B, C + (1 << 20))])
     assert emb.emb_qlayer_seq_workspace(chain, 1) == 0
     assert emb.emb_qlayer_seq_workspace(chain, 816) == 0
+
+
+def test_seq_rejects_misaligned_workspace(L):
+    """A workspace must be 256-byte aligned; checked before anything is enqueued."""
+    chain = _layers([(0, A, 128, 64, B, C)])
+    assert L.emb_qlayer_seq(chain, 1, 1, ctypes.c_void_p(B + (8 << 20) + 16), 1 << 20, None) == emb.EMB_EALIGN
+    h = ctypes.c_void_p()
+    assert L.emb_chain_create(chain, 1, 1, ctypes.c_void_p(B + (8 << 20) + 16), 1 << 20,
+                              ctypes.byref(h)) == emb.EMB_EALIGN
+    assert h.value is None
 
 
 def test_precise_operand_flag(L):

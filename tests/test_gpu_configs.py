@@ -1,6 +1,7 @@
 """Parity at the full sizes of every workload (one closed-loop step of the paper's
 batch-1 setting: decode M=1, action chunk M=50, prefill M=280/768/816), run through
-emb_qlayer_seq exactly as the bench launches it. Every linear is checked on sampled
+emb_qlayer_seq exactly as the bench launches it (with the workspace its recorded chains
+get, so prefill layers take the stream-K schedule where it pays). Every linear is checked on sampled
 output rows (the oracle quantises those rows of W itself and computes them one by
 one); layer 0 of each distinct shape is also compared in full."""
 import numpy as np
@@ -36,8 +37,12 @@ def _run_workload(w: wl.Workload, rows_per_linear=12, full_first=True, layers=No
             checks.append((lin, rows, Wrows, Xb, img, Y, full))
             specs.append((w.fmt, img, lin.N, lin.K, X, Y))
             del W
-    emb.emb_qlayer_seq(specs, w.M)
+    # with the workspace the bench's recorded chains take (stream-K prefill launches)
+    ws = emb.chain_workspace(specs, w.M)
+    emb.emb_qlayer_seq(specs, w.M, ws, 0 if ws is None else ws.numel())
     assert emb.emb_device_status() == emb.EMB_OK
+    if ws is not None:
+        assert int(ws[:4096].count_nonzero()) == 0, "stream-K flags left set"
     worst = 0.0
     toks = np.arange(w.M) if token_sample is None else token_sample
     for lin, rows, Wrows, Xb, img, Y, full in checks:
