@@ -228,6 +228,19 @@ EMB_API emb_status emb_qlayer_seq(const emb_qlayer* layers, int n_layers, int64_
 EMB_API emb_status emb_qlayer_seq_chained(const emb_qlayer* layers, int n_layers, int64_t M,
                                           emb_stream_t stream);
 
+/* Section 3.2, principle 2 has the caller own every buffer of a chain; this call is the
+ * exception and has no counterpart in the paper. emb_qlayer_seq with a workspace that the
+ * library owns: a static device array of 48 MB (zero at load) in this library's module on
+ * each device, so a chain needs no allocation by the caller and still takes its stream-K
+ * schedules (a chain wanting more than 48 MB runs as with a NULL workspace). Results are
+ * bitwise those of emb_qlayer_seq with a caller workspace. Each call first zeroes the
+ * array's 4 KB of flags on `stream` when a launch of the chain will use it. The array is
+ * one per device: calls on different streams of one device must not run concurrently
+ * (order them, e.g. with events); recording the call into a graph records the array's
+ * address. Errors as emb_qlayer_seq; EMB_ECUDA if the array cannot be reached. */
+EMB_API emb_status emb_qlayer_seq_noalloc(const emb_qlayer* layers, int n_layers, int64_t M,
+                                          emb_stream_t stream);
+
 /* ------------------------------------------------------------ recorded chains
  * Graph replay and buffer reuse (Section 3.2, design principle 2): the
  * launches that emb_qlayer_seq(layers, n_layers, M, workspace, ws_bytes, ...) enqueues

@@ -106,6 +106,8 @@ def lib():
     L.emb_build_info.restype = ctypes.c_char_p
     L.emb_qlayer_seq_chained.argtypes = [ctypes.POINTER(emb_qlayer), i32, i64, vp]
     L.emb_qlayer_seq_chained.restype = i32
+    L.emb_qlayer_seq_noalloc.argtypes = [ctypes.POINTER(emb_qlayer), i32, i64, vp]
+    L.emb_qlayer_seq_noalloc.restype = i32
     L.emb_chain_record_begin.argtypes = [vp]
     L.emb_chain_record_begin.restype = i32
     L.emb_chain_record_end.argtypes = [vp, ctypes.POINTER(vp)]
@@ -219,6 +221,13 @@ def emb_qlayer_seq_chained(layers, M: int, stream=None) -> None:
     (the call's weights must not be written by that launch)."""
     arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
     _check(lib().emb_qlayer_seq_chained(arr, len(arr), M, _stream(stream)), "emb_qlayer_seq_chained")
+
+
+def emb_qlayer_seq_noalloc(layers, M: int, stream=None) -> None:
+    """emb_qlayer_seq with the library's own static device workspace (one per device;
+    calls on different streams of a device must not overlap)."""
+    arr = layers if isinstance(layers, ctypes.Array) else make_layers(layers)
+    _check(lib().emb_qlayer_seq_noalloc(arr, len(arr), M, _stream(stream)), "emb_qlayer_seq_noalloc")
 
 
 def emb_chain_create(layers, M: int, workspace=None, ws_bytes: int = 0) -> int:

@@ -18,6 +18,10 @@ namespace {
 
 __device__ int g_status_word;  // OR of kStatus* flags; read and cleared by emb_device_status
 __device__ int g_status_read;  // where emb_device_status's exchange leaves the value it read
+// emb_qlayer_seq_noalloc's workspace: the library's own, zero at module load (4 KB of
+// flags, then the partial tiles of one stream-K launch: room for ~190 SMs at the largest tile)
+constexpr size_t kScratchBytes = size_t(48) << 20;
+__device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
 // Token counts up to this run the GEMV; above it, the tensor-core GEMM.
 constexpr int64_t kGemvMaxM = 4;
@@ -33,6 +37,16 @@ int* status_ptr() {
         if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
         ptrs[dev] = static_cast<int*>(p);
     }
+    return ptrs[dev];
+}
+
+void* scratch_ptr() {
+    static std::mutex mu;
+    static void* ptrs[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!ptrs[dev] && cudaGetSymbolAddress(&ptrs[dev], g_scratch) != cudaSuccess) ptrs[dev] = nullptr;
     return ptrs[dev];
 }
 
@@ -323,6 +337,26 @@ emb_status emb_qlayer_seq_chained(const emb_qlayer* layers, int n_layers, int64_
     const emb_status st = prepare_seq(layers, n_layers, M, refs);
     if (st != EMB_OK) return st;
     return enqueue_seq(refs, reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+emb_status emb_qlayer_seq_noalloc(const emb_qlayer* layers, int n_layers, int64_t M,
+                                  emb_stream_t stream) {
+    std::vector<GroupRef> refs;
+    emb_status st = prepare_seq(layers, n_layers, M, refs);
+    if (st != EMB_OK) return st;
+    size_t need = 0;
+    if (M > kGemvMaxM)
+        for (const GroupRef& g : refs) need = std::max(need, gemm_tc_workspace(g));
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (need > 0 && need <= kScratchBytes) {
+        void* ws = scratch_ptr();
+        if (!ws) return EMB_ECUDA;
+        // the flags start at zero whatever an earlier call left (e.g. after EMB_ETIMEOUT)
+        if (cudaMemsetAsync(ws, 0, 4096, s) != cudaSuccess) return EMB_ECUDA;
+        st = attach_workspace(refs, M, ws, kScratchBytes);
+        if (st != EMB_OK) return st;
+    }
+    return enqueue_seq(refs, s, false);
 }
 
 }  // extern "C"
