@@ -183,6 +183,7 @@ GEMV_CASES = [
     (emb.EMB_Q8_0, 6144, 2048, 1, "staged", "all"),
     (emb.EMB_Q8_0, 6144, 2048, 4, "staged MT=4", "all"),
     (emb.EMB_Q4_0, 12288, 2048, 1, "staged", "all"),
+    (emb.EMB_Q4_0, 4096, 12288, 1, "staged, 6 KB rows", "spread"),
     (emb.EMB_Q6_0, 8192, 2048, 1, "staged", "all"),
     (emb.EMB_Q6_0, 8192, 2048, 2, "staged MT=2", "all"),
     # Q4_0 mma.sync kernel: >= 12 MB, rows <= 2 KB, M = 2..4
