@@ -224,6 +224,9 @@ GEMM_CASES = [
     # prefill: one 208-token tile per CTA (M = 816)
     (emb.EMB_Q8_0, 2048, 2048, 816, "M=816 one tile per CTA", "spread"),
     (emb.EMB_Q6_0, 2048, 2048, 816, "M=816 one tile per CTA", "spread"),
+    # prefill with more tiles than SMs: persistent CTAs looping over (weight, token) tiles
+    (emb.EMB_Q8_0, 10240, 1024, 816, "M=816 persistent CTAs", "spread"),
+    (emb.EMB_Q4_0, 10240, 1024, 816, "M=816 persistent CTAs", "spread"),
 ]
 
 
