@@ -293,6 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
     }
     if (warp == 1) {
+        // all 512 columns: one CTA per SM (see ptx::tmem_alloc for why this never waits)
         ptx::tmem_alloc(tmem_slot, p.tmem_cols);
         ptx::tmem_relinquish();
     }

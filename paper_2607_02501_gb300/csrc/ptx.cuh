@@ -212,6 +212,11 @@ __device__ __forceinline__ float4 ld_dsmem_f32x4(uint32_t caddr) {
 }
 
 // -------------------------------------------------------------------- tcgen05
+// tcgen05.alloc blocks until ncols columns are free on the SM; it is the one wait in the
+// library without a time limit. It cannot block here because no two CTAs that allocate
+// share an SM: every GEMM CTA asks for all 512 columns and its dynamic shared memory is
+// padded above half of the SM's (gemm_tc.cu, kOneCtaPerSm), and no other kernel of the
+// library allocates tensor memory. A variant with two CTAs per SM must keep each below 256.
 __device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(dst_smem)),
