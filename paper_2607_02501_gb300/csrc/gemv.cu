@@ -252,9 +252,10 @@ cudaError_t launch_one(const GemvParams& p, int grid_x, int grid_y, bool pdl, cu
 template <int FMT, int R, int NT>
 cudaError_t dispatch_mt(const GemvParams& p, int grid_x, int M, bool pdl, cudaStream_t s) {
     // Q8_0 rows longer than one pass of the CTA's threads (at most four) are loaded whole
-    // before the wait (measured on GB300, Gemma-2B decode chain at M = 1, whose down
-    // projection 2048 x 16384 takes this path: Q8_0 3899 -> 3987 GB/s). Not for Q4_0:
-    // its variant needs ~100 registers, halves the resident CTAs and lost (2265 -> 2068).
+    // before the wait (measured on GB300 on the Gemma-2B decode chain at M = 1, whose down
+    // projection 2048 x 16384 took this path before the hybrid kernel: Q8_0 3899 -> 3987
+    // GB/s). Not for Q4_0: its variant needs ~100 registers, halves the resident CTAs and
+    // lost (2265 -> 2068).
     if constexpr (FMT == EMB_Q8_0 && R <= 2) {
         if (M == 1 && p.U > NT && p.U <= 4 * NT) return launch_one<FMT, R, NT, 1, 4>(p, grid_x, 1, pdl, s);
     }
@@ -840,6 +841,217 @@ bool launch_q4_mma(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     return true;
 }
 
+// ------------------------------------------------------------------ hybrid GEMV
+// Long rows at M = 1 (more than one pass of the CTA's threads; Gemma-2B's down projection,
+// 2048 x 16384). The register kernel can keep only as many bytes in flight as the CTAs
+// resident on an SM hold in registers, so such a matrix streams in two waves of CTAs whose
+// loads do not overlap. Here a CTA owns four rows: its threads load their units of the first
+// two straight into registers and one thread bulk-copies the other two rows (codes and
+// scales) into shared memory, all before griddepcontrol.wait. With the same registers a CTA
+// has twice the bytes in flight, and one wave of CTAs requests the whole matrix. Each row's
+// sum is formed as in the register kernel: per thread over its units in order, over the
+// lanes by a shuffle tree, over the warps in order.
+constexpr int kHybThreads = 256;
+constexpr int kHybHeader = 256;  // mbarrier (0..7), cross-warp sums [8 warps][4 rows] (16..143)
+
+struct HybridParams {
+    const uint8_t* codes[kMaxGroup];
+    const __half* scales[kMaxGroup];
+    void* Y[kMaxGroup];
+    int32_t N[kMaxGroup];
+    int32_t tile0[kMaxGroup + 1];  // first four-row tile of each matrix (prefix sums)
+    int32_t n_mats;
+    int32_t K, ldS, U;
+    int32_t epi;
+    const __nv_bfloat16* X;
+    int* status;
+};
+
+template <int FMT, int PF>
+__global__ void __launch_bounds__(kHybThreads, 4) gemv_hybrid_kernel(const __grid_constant__ HybridParams p) {
+    constexpr int UW = (FMT == EMB_Q8_0) ? 16 : 32;
+    constexpr int NT = kHybThreads, NWARP = NT / 32;
+    extern __shared__ __align__(128) uint8_t smem[];
+    uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
+    float* red = reinterpret_cast<float*>(smem + 16);  // [NWARP][4]
+    const int tile = blockIdx.x;
+    int g = 0;
+#pragma unroll
+    for (int i = 1; i < kMaxGroup; ++i)
+        if (i < p.n_mats && tile >= p.tile0[i]) g = i;
+    const int N = p.N[g];
+    const int row0 = (tile - p.tile0[g]) * 4;
+    const int t = threadIdx.x;
+    const int U = p.U;
+    const int64_t row_bytes = (FMT == EMB_Q8_0) ? int64_t(p.K) : int64_t(p.K) / 2;
+    const int ns = min(2, max(0, N - (row0 + 2)));  // rows row0 + 2, row0 + 3 in shared memory
+    uint8_t* codes_s = smem + kHybHeader;           // [2][row_bytes]
+    uint8_t* scales_b = codes_s + 2 * row_bytes;    // [2][ldS] fp16
+    const __half* scales_s = reinterpret_cast<const __half*>(scales_b);
+
+    if (t == 0) {
+        ptx::mbar_init(bar, 1);
+        ptx::fence_mbar_init();
+        if (ns > 0) {
+            // row_bytes and ldS * 2 are multiples of 16: both copies are 16-byte aligned
+            const uint32_t cb = uint32_t(ns) * uint32_t(row_bytes), sb = uint32_t(ns) * uint32_t(p.ldS) * 2u;
+            ptx::mbar_arrive_expect_tx(bar, cb + sb);
+            ptx::bulk_load(codes_s, p.codes[g] + int64_t(row0 + 2) * row_bytes, cb, bar);
+            ptx::bulk_load(scales_b, p.scales[g] + int64_t(row0 + 2) * p.ldS, sb, bar);
+        }
+        // the activation row towards L2 while the previous launch finishes (one CTA asks)
+        if (blockIdx.x == 0) ptx::prefetch_l2(p.X, uint32_t(p.K) * 2u);
+    }
+    griddep_launch_dependents();
+
+    // the register rows: every unit of this thread, loaded before the dependency wait
+    const uint8_t* cbase = p.codes[g] + int64_t(row0) * row_bytes;
+    const __half* sbase = p.scales[g] + int64_t(row0) * p.ldS;
+    uint4 cp[PF][2];
+    float dp[PF][2];
+#pragma unroll
+    for (int k = 0; k < PF; ++k) {
+        const int uk = t + k * NT;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            if (uk < U && row0 + r < N) {
+                cp[k][r] = ld_stream_u4(cbase + r * row_bytes + int64_t(uk) * 16);
+                dp[k][r] = __half2float(sbase[int64_t(r) * p.ldS + ((FMT == EMB_Q8_0) ? (uk >> 1) : uk)]);
+            } else {
+                cp[k][r] = make_uint4(0, 0, 0, 0);
+                dp[k][r] = 0.0f;
+            }
+        }
+    }
+    __syncthreads();  // the barrier's initialisation is visible to every waiting thread
+    // weights do not depend on earlier launches; X and Y may
+    griddep_wait();
+    // bounded wait; the CTA leaves together if any of its threads gave up
+    const bool ok = ns == 0 || ptx::mbar_wait(bar, 0, nullptr, p.status, kWaitLimitNs);
+    if (__syncthreads_or(!ok)) return;
+
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    const uint2 h0 = make_uint2(0, 0);
+#pragma unroll
+    for (int k = 0; k < PF; ++k) {
+        const int uk = t + k * NT;
+        if (uk >= U) break;
+        float x[UW];
+        const uint4* xp = reinterpret_cast<const uint4*>(p.X + int64_t(uk) * UW);
+#pragma unroll
+        for (int v = 0; v < UW / 8; ++v) {
+            const uint4 hx = xp[v];
+            x[8 * v + 0] = lo_bf16(hx.x); x[8 * v + 1] = hi_bf16(hx.x);
+            x[8 * v + 2] = lo_bf16(hx.y); x[8 * v + 3] = hi_bf16(hx.y);
+            x[8 * v + 4] = lo_bf16(hx.z); x[8 * v + 5] = hi_bf16(hx.z);
+            x[8 * v + 6] = lo_bf16(hx.w); x[8 * v + 7] = hi_bf16(hx.w);
+        }
+#pragma unroll
+        for (int r = 0; r < 2; ++r) acc[r] = fmaf(dp[k][r], dot_unit<FMT>(cp[k][r], h0, x), acc[r]);
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            if (r < ns) {
+                const uint4 c = *reinterpret_cast<const uint4*>(codes_s + r * row_bytes + int64_t(uk) * 16);
+                const float d = __half2float(scales_s[r * p.ldS + ((FMT == EMB_Q8_0) ? (uk >> 1) : uk)]);
+                acc[2 + r] = fmaf(d, dot_unit<FMT>(c, h0, x), acc[2 + r]);
+            }
+        }
+    }
+
+    const int lane = t & 31, warp = t >> 5;
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        float v = acc[r];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) red[warp * 4 + r] = v;
+    }
+    __syncthreads();
+    if (p.epi >= EMB_EPI_GEGLU) {
+        // gate row row0 + 2i and up row row0 + 2i + 1
+        if (t < 2) {
+            float gate = 0.0f, up = 0.0f;
+#pragma unroll
+            for (int w = 0; w < NWARP; ++w) {
+                gate += red[w * 4 + 2 * t];
+                up += red[w * 4 + 2 * t + 1];
+            }
+            const int n = row0 + 2 * t;
+            if (n < N) epi_store_gated(p.epi, p.Y[g], 0, n, N, gate, up);
+        }
+    } else if (t < 4) {
+        float v = 0.0f;
+#pragma unroll
+        for (int w = 0; w < NWARP; ++w) v += red[w * 4 + t];
+        const int n = row0 + t;
+        if (n < N) epi_store(p.epi, p.Y[g], 0, n, N, v);
+    }
+}
+
+template <int FMT, int PF>
+cudaError_t launch_hybrid_one(const HybridParams& p, int tiles, size_t smem, bool pdl, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(tiles, 1, 1);
+    cfg.blockDim = dim3(kHybThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    if (smem > 48 * 1024) {
+        const cudaError_t e = cudaFuncSetAttribute(gemv_hybrid_kernel<FMT, PF>,
+                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        if (e != cudaSuccess) return e;
+    }
+    return cudaLaunchKernelEx(&cfg, gemv_hybrid_kernel<FMT, PF>, p);
+}
+
+// Which layers take the hybrid path: M = 1, Q8_0 or Q4_0, rows longer than the staged path
+// takes at M = 1 and than one pass of 256 threads (2..4 units per thread), matrices of at
+// least kStageMinBytes. Measured on GB300 (graph-replayed chains of the Gemma-2B down
+// projection, 2048 x 16384, each launch its own weights; register kernel -> hybrid):
+// Q8_0 9.76 -> 9.54 us, Q4_0 9.75 -> 9.65 us.
+bool launch_hybrid(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
+    if (g.M != 1 || (g.fmt != EMB_Q8_0 && g.fmt != EMB_Q4_0)) return false;
+    const int64_t row_bytes = (g.fmt == EMB_Q8_0) ? g.K : g.K / 2;
+    const int64_t U = (g.fmt == EMB_Q8_0) ? g.K / 16 : g.K / 32;
+    if (row_bytes <= kStageMaxRowBytesM1 || U <= kHybThreads || U > 4 * kHybThreads) return false;
+    int64_t rows = 0;
+    for (int i = 0; i < g.n_mats; ++i) rows += g.mats[i].N;
+    if (rows * row_bytes < kStageMinBytes) return false;
+    HybridParams p = {};
+    int tiles = 0;
+    for (int i = 0; i < g.n_mats; ++i) {
+        p.codes[i] = g.mats[i].codes;
+        p.scales[i] = g.mats[i].scales;
+        p.Y[i] = g.mats[i].Y;
+        p.N[i] = int32_t(g.mats[i].N);
+        p.tile0[i] = tiles;
+        tiles += int((g.mats[i].N + 3) / 4);
+    }
+    p.tile0[g.n_mats] = tiles;
+    p.n_mats = g.n_mats;
+    p.K = int32_t(g.K);
+    p.ldS = int32_t(g.ldS);
+    p.U = int32_t(U);
+    p.epi = g.epi;
+    p.X = g.X;
+    p.status = status;
+    const size_t smem = kHybHeader + size_t(2) * size_t(row_bytes + g.ldS * 2);
+    const int pf = int((U + kHybThreads - 1) / kHybThreads);
+    if (g.fmt == EMB_Q8_0)
+        err = pf == 2 ? launch_hybrid_one<EMB_Q8_0, 2>(p, tiles, smem, pdl, s)
+            : pf == 3 ? launch_hybrid_one<EMB_Q8_0, 3>(p, tiles, smem, pdl, s)
+                      : launch_hybrid_one<EMB_Q8_0, 4>(p, tiles, smem, pdl, s);
+    else
+        err = pf == 2 ? launch_hybrid_one<EMB_Q4_0, 2>(p, tiles, smem, pdl, s)
+            : pf == 3 ? launch_hybrid_one<EMB_Q4_0, 3>(p, tiles, smem, pdl, s)
+                      : launch_hybrid_one<EMB_Q4_0, 4>(p, tiles, smem, pdl, s);
+    return true;
+}
+
 }  // namespace
 
 cudaError_t launch_gemv_regs(const GroupRef& g, bool pdl, cudaStream_t s);
@@ -848,6 +1060,7 @@ cudaError_t launch_gemv(const GroupRef& g, bool pdl, int* status, cudaStream_t s
     cudaError_t err = cudaSuccess;
     if (launch_q4_mma(g, pdl, status, s, err)) return err;
     if (launch_staged(g, pdl, status, s, err)) return err;
+    if (launch_hybrid(g, pdl, status, s, err)) return err;
     return launch_gemv_regs(g, pdl, s);
 }
 

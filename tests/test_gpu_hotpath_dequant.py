@@ -102,13 +102,16 @@ def run_onehot(fmt: int, img_dev: torch.Tensor, N: int, K: int, M: int, ks) -> n
     what is left); row p of the result is the call's output for activation e_{ks[p]}."""
     X = onehot_rows(ks, K)
     P = len(ks)
-    Y = torch.full((P, N), float("nan"), dtype=torch.float32, device="cuda")
+    # one-token calls write one row each: a row pitch of a multiple of four floats keeps
+    # every call's output 16-byte aligned whatever N is
+    pitch = (N + 3) // 4 * 4 if M == 1 else N
+    Y = torch.full((P, pitch), float("nan"), dtype=torch.float32, device="cuda")
     for j in range(0, P, M):
         m = min(M, P - j)
         emb.emb_qmatmul(fmt, img_dev, X[j].data_ptr(), Y[j].data_ptr(), m, N, K)
     torch.cuda.synchronize()
     assert emb.emb_device_status() == emb.EMB_OK
-    return Y.cpu().numpy()
+    return Y[:, :N].cpu().numpy()
 
 
 def _assert_columns_equal(Y: np.ndarray, W: np.ndarray, ks, what: str) -> None:
@@ -173,12 +176,18 @@ GEMV_CASES = [
     # four rows per CTA (2048 rows, 16-byte units per row < 320)
     (emb.EMB_Q4_0, 2048, 2048, 1, "register R=4", "all"),
     (emb.EMB_Q8_0, 2048, 2048, 2, "register R=4 MT=2", "all"),
-    # long Q8_0 rows: a thread's whole row share loaded before the wait (PF = 4), one and
-    # two rows per CTA; the Gemma-2B down projection shape
+    # long Q8_0 rows below 12 MB: a thread's whole row share loaded before the wait (PF = 4)
     (emb.EMB_Q8_0, 256, 16384, 1, "register PF=4 R=1", "spread"),
-    (emb.EMB_Q8_0, 2048, 16384, 1, "register PF=4 R=2", "spread"),
-    (emb.EMB_Q4_0, 2048, 16384, 1, "register R=2 long rows", "spread"),
     (emb.EMB_Q6_0, 2048, 16384, 1, "register R=2 long rows", "spread"),
+    # hybrid kernel (rows > 6 KB, >= 12 MB, M = 1): two rows per CTA in registers, two in
+    # shared memory; the Gemma-2B down projection shape, 2..4 units per thread, and ragged
+    # row counts (the last CTA with one or no shared-memory row)
+    (emb.EMB_Q8_0, 2048, 16384, 1, "hybrid PF=4", "spread"),
+    (emb.EMB_Q4_0, 2048, 16384, 1, "hybrid PF=2", "spread"),
+    (emb.EMB_Q8_0, 2048, 8192, 1, "hybrid PF=2", "spread"),
+    (emb.EMB_Q8_0, 1027, 12288, 1, "hybrid PF=3, one smem row in the last CTA", "spread"),
+    (emb.EMB_Q4_0, 1024, 24576, 1, "hybrid PF=3", "spread"),
+    (emb.EMB_Q4_0, 1538, 16384, 1, "hybrid, no smem row in the last CTA", "spread"),
     # staged kernel: >= 12 MB of codes with rows <= 6 KB at M = 1; any rows at M = 2..4
     (emb.EMB_Q8_0, 6144, 2048, 1, "staged", "all"),
     (emb.EMB_Q8_0, 6144, 2048, 4, "staged MT=4", "all"),
