@@ -57,10 +57,11 @@ def test_workspace_wanted_only_where_tiles_leave_sms_idle(cuda_device):
 @pytest.mark.parametrize("fmt,M,N,K", CASES)
 def test_streamk_parity(cuda_device, fmt, M, N, K):
     W, Xb, img, X = _setup(fmt, M, N, K, 11 + N + K)
-    n = emb.emb_qlayer_seq_workspace([(fmt, img, N, K, X, torch.empty(1, device="cuda"))], M)
+    Y = torch.full((M, N), float("nan"), device="cuda")
+    # (the query validates the layer as a call would: Y must be a real [M][N] buffer)
+    n = emb.emb_qlayer_seq_workspace([(fmt, img, N, K, X, Y)], M)
     assert n > 0, "this shape should take the stream-K schedule"
     ws = torch.zeros(n, dtype=torch.uint8, device="cuda")
-    Y = torch.full((M, N), float("nan"), device="cuda")
     _run(fmt, img, X, Y, M, N, K, ws)
     assert int(ws[:4096].count_nonzero()) == 0, "ready flags left set"
     Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
