@@ -525,7 +525,7 @@ def measure_workload(name, ws, args, dev, dist, steps, warmup, e2e_steps, clocks
                     "peak_source": f"{peaks['source']} HBM copy bandwidth"}
         roof["frac"] = roof["achieved"] / roof["peak"]
         roof["traffic"] = kernel_traffic(name, c["w"])
-        roof["kernel"] = ("GEMV (gemv_staged_kernel + gemv_hybrid_kernel + gemv_kernel + gemv_q4_mma_kernel)" if c["w"].M <= 4
+        roof["kernel"] = ("GEMV (gemv_staged_kernel + gemv_ring_kernel + gemv_kernel + gemv_q4_mma_kernel)" if c["w"].M <= 4
                           else "gemm_tc_kernel") + f" <{wl.FMT_NAMES[c['w'].fmt]}>"
         roof["launches_per_step"] = c["launches"] * c["w"].repeats
         roof["per_launch_us"] = per_launch_ms * 1e3

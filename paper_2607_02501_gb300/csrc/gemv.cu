@@ -22,6 +22,7 @@
 // (coherent, L1-cached) loads and Y written only after it: the previous launch may have
 // just written X, and after griddepcontrol.wait its writes are visible to ordinary loads.
 // Up to kMaxGroup matrices that read the same X (q/k/v or gate/up) share one launch.
+#include <algorithm>
 #include <mutex>
 
 #include "dequant_dot.cuh"
@@ -253,7 +254,7 @@ template <int FMT, int R, int NT>
 cudaError_t dispatch_mt(const GemvParams& p, int grid_x, int M, bool pdl, cudaStream_t s) {
     // Q8_0 rows longer than one pass of the CTA's threads (at most four) are loaded whole
     // before the wait (measured on GB300 on the Gemma-2B decode chain at M = 1, whose down
-    // projection 2048 x 16384 took this path before the hybrid kernel: Q8_0 3899 -> 3987
+    // projection 2048 x 16384 took this path before the ring kernel: Q8_0 3899 -> 3987
     // GB/s). Not for Q4_0: its variant needs ~100 registers, halves the resident CTAs and
     // lost (2265 -> 2068).
     if constexpr (FMT == EMB_Q8_0 && R <= 2) {
@@ -841,158 +842,185 @@ bool launch_q4_mma(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     return true;
 }
 
-// ------------------------------------------------------------------ hybrid GEMV
-// Long rows at M = 1 (more than one pass of the CTA's threads; Gemma-2B's down projection,
-// 2048 x 16384). The register kernel can keep only as many bytes in flight as the CTAs
-// resident on an SM hold in registers, so such a matrix streams in two waves of CTAs whose
-// loads do not overlap. Here a CTA owns four rows: its threads load their units of the first
-// two straight into registers and one thread bulk-copies the other two rows (codes and
-// scales) into shared memory, all before griddepcontrol.wait. With the same registers a CTA
-// has twice the bytes in flight, and one wave of CTAs requests the whole matrix. Each row's
-// sum is formed as in the register kernel: per thread over its units in order, over the
-// lanes by a shuffle tree, over the warps in order.
-constexpr int kHybThreads = 256;
-constexpr int kHybHeader = 256;  // mbarrier (0..7), cross-warp sums [8 warps][4 rows] (16..143)
+// ------------------------------------------------------------------ ring GEMV
+// Long rows at M = 1 (more than one pass of 256 threads; Gemma-2B's down projection,
+// 2048 x 16384). The register kernel holds only as many bytes in flight as the resident
+// CTAs' registers, so such a matrix streams in two waves of CTAs whose loads do not overlap,
+// and the staged kernel re-stages the whole activation row for every tile of one or two
+// rows. Here a CTA owns a run of consecutive rows (crossing
+// matrix boundaries within the group) and keeps the activation row it needs in registers:
+// each thread's units t + k*256 of X, loaded once after griddepcontrol.wait and reused for
+// every row. The rows stream through a ring of shared-memory stages (one row of codes and
+// its scales each; as many as kRingBudget holds, 2..8), filled by bulk copies that one
+// thread issues -- a ring's worth before the wait -- and refills as soon as all eight warps
+// have released a stage. The warps run on the ring's barriers alone (no CTA-wide barrier
+// until the reduction). Each row is summed as in the register kernel (per thread over its
+// units in order, shuffle tree, warps in order), so its bits equal that kernel's.
+constexpr int kRingThreads = 256;
+constexpr int kRingMaxStages = 8;
+constexpr int kRingBudget = 56 * 1024;  // ring bytes per CTA: stages = budget / stage, 2..8
+constexpr int kRingFlush = 16;  // rows whose per-warp sums are kept before a CTA-wide reduction
+// barriers (0..127), abort flag (128), per-warp sums (144..655), then the ring
+constexpr int kRingHeader = 144 + kRingFlush * (kRingThreads / 32) * 4;
 
-struct HybridParams {
+struct RingParams {
     const uint8_t* codes[kMaxGroup];
     const __half* scales[kMaxGroup];
     void* Y[kMaxGroup];
     int32_t N[kMaxGroup];
-    int32_t tile0[kMaxGroup + 1];  // first four-row tile of each matrix (prefix sums)
+    int32_t row0[kMaxGroup + 1];  // first row of each matrix in the group's row order
     int32_t n_mats;
     int32_t K, ldS, U;
+    int32_t rows_per_cta, rows_total;
+    int32_t stage_bytes;          // one row of codes + its scales, rounded up to 16
+    int32_t stages;               // ring depth (2..kRingMaxStages)
     int32_t epi;
     const __nv_bfloat16* X;
     int* status;
 };
 
 template <int FMT, int PF>
-__global__ void __launch_bounds__(kHybThreads, 4) gemv_hybrid_kernel(const __grid_constant__ HybridParams p) {
+__global__ void __launch_bounds__(kRingThreads, 2) gemv_ring_kernel(const __grid_constant__ RingParams p) {
     constexpr int UW = (FMT == EMB_Q8_0) ? 16 : 32;
-    constexpr int NT = kHybThreads, NWARP = NT / 32;
+    constexpr int NT = kRingThreads, NWARP = NT / 32;
     extern __shared__ __align__(128) uint8_t smem[];
-    uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
-    float* red = reinterpret_cast<float*>(smem + 16);  // [NWARP][4]
-    const int tile = blockIdx.x;
-    int g = 0;
-#pragma unroll
-    for (int i = 1; i < kMaxGroup; ++i)
-        if (i < p.n_mats && tile >= p.tile0[i]) g = i;
-    const int N = p.N[g];
-    const int row0 = (tile - p.tile0[g]) * 4;
-    const int t = threadIdx.x;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem);              // [stages]
+    uint64_t* empty = full + kRingMaxStages;                          // [stages]
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + 128);  // a wait gave up
+    float* red = reinterpret_cast<float*>(smem + 144);               // [kRingFlush][NWARP]
+    uint8_t* ring = smem + kRingHeader;                               // [stages][stage_bytes]
+    const int S = p.stages;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int U = p.U;
     const int64_t row_bytes = (FMT == EMB_Q8_0) ? int64_t(p.K) : int64_t(p.K) / 2;
-    const int ns = min(2, max(0, N - (row0 + 2)));  // rows row0 + 2, row0 + 3 in shared memory
-    uint8_t* codes_s = smem + kHybHeader;           // [2][row_bytes]
-    uint8_t* scales_b = codes_s + 2 * row_bytes;    // [2][ldS] fp16
-    const __half* scales_s = reinterpret_cast<const __half*>(scales_b);
-
+    const int r_begin = blockIdx.x * p.rows_per_cta;
+    const int n_rows = min(p.rows_per_cta, p.rows_total - r_begin);
+    // global row -> (matrix, row within it)
+    auto locate = [&](int gr, int& g, int& n) {
+        g = 0;
+#pragma unroll
+        for (int i = 1; i < kMaxGroup; ++i)
+            if (i < p.n_mats && gr >= p.row0[i]) g = i;
+        n = gr - p.row0[g];
+    };
+    auto issue = [&](int i, int stage) {  // row i of this CTA into a stage
+        int g, n;
+        locate(r_begin + i, g, n);
+        uint8_t* st = ring + stage * p.stage_bytes;
+        uint64_t* bar = &full[stage];
+        const uint32_t cb = uint32_t(row_bytes), sb = uint32_t(p.ldS) * 2u;
+        ptx::mbar_arrive_expect_tx(bar, cb + sb);
+        ptx::bulk_load(st, p.codes[g] + int64_t(n) * row_bytes, cb, bar);
+        ptx::bulk_load(st + row_bytes, p.scales[g] + int64_t(n) * p.ldS, sb, bar);
+    };
     if (t == 0) {
-        ptx::mbar_init(bar, 1);
-        ptx::fence_mbar_init();
-        if (ns > 0) {
-            // row_bytes and ldS * 2 are multiples of 16: both copies are 16-byte aligned
-            const uint32_t cb = uint32_t(ns) * uint32_t(row_bytes), sb = uint32_t(ns) * uint32_t(p.ldS) * 2u;
-            ptx::mbar_arrive_expect_tx(bar, cb + sb);
-            ptx::bulk_load(codes_s, p.codes[g] + int64_t(row0 + 2) * row_bytes, cb, bar);
-            ptx::bulk_load(scales_b, p.scales[g] + int64_t(row0 + 2) * p.ldS, sb, bar);
+        *abort_flag = 0;
+        for (int i = 0; i < S; ++i) {
+            ptx::mbar_init(&full[i], 1);
+            ptx::mbar_init(&empty[i], NWARP);
         }
+        ptx::fence_mbar_init();
+        for (int i = 0; i < S && i < n_rows; ++i) issue(i, i);
         // the activation row towards L2 while the previous launch finishes (one CTA asks)
         if (blockIdx.x == 0) ptx::prefetch_l2(p.X, uint32_t(p.K) * 2u);
     }
     griddep_launch_dependents();
-
-    // the register rows: every unit of this thread, loaded before the dependency wait
-    const uint8_t* cbase = p.codes[g] + int64_t(row0) * row_bytes;
-    const __half* sbase = p.scales[g] + int64_t(row0) * p.ldS;
-    uint4 cp[PF][2];
-    float dp[PF][2];
-#pragma unroll
-    for (int k = 0; k < PF; ++k) {
-        const int uk = t + k * NT;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            if (uk < U && row0 + r < N) {
-                cp[k][r] = ld_stream_u4(cbase + r * row_bytes + int64_t(uk) * 16);
-                dp[k][r] = __half2float(sbase[int64_t(r) * p.ldS + ((FMT == EMB_Q8_0) ? (uk >> 1) : uk)]);
-            } else {
-                cp[k][r] = make_uint4(0, 0, 0, 0);
-                dp[k][r] = 0.0f;
-            }
-        }
-    }
-    __syncthreads();  // the barrier's initialisation is visible to every waiting thread
+    __syncthreads();  // the barriers' initialisation is visible to every waiting thread
     // weights do not depend on earlier launches; X and Y may
     griddep_wait();
-    // bounded wait; the CTA leaves together if any of its threads gave up
-    const bool ok = ns == 0 || ptx::mbar_wait(bar, 0, nullptr, p.status, kWaitLimitNs);
-    if (__syncthreads_or(!ok)) return;
-
-    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-    const uint2 h0 = make_uint2(0, 0);
+    float x[PF][UW];
 #pragma unroll
     for (int k = 0; k < PF; ++k) {
         const int uk = t + k * NT;
-        if (uk >= U) break;
-        float x[UW];
-        const uint4* xp = reinterpret_cast<const uint4*>(p.X + int64_t(uk) * UW);
+        const uint4* xp = reinterpret_cast<const uint4*>(p.X + int64_t(min(uk, U - 1)) * UW);
 #pragma unroll
         for (int v = 0; v < UW / 8; ++v) {
             const uint4 hx = xp[v];
-            x[8 * v + 0] = lo_bf16(hx.x); x[8 * v + 1] = hi_bf16(hx.x);
-            x[8 * v + 2] = lo_bf16(hx.y); x[8 * v + 3] = hi_bf16(hx.y);
-            x[8 * v + 4] = lo_bf16(hx.z); x[8 * v + 5] = hi_bf16(hx.z);
-            x[8 * v + 6] = lo_bf16(hx.w); x[8 * v + 7] = hi_bf16(hx.w);
+            x[k][8 * v + 0] = lo_bf16(hx.x); x[k][8 * v + 1] = hi_bf16(hx.x);
+            x[k][8 * v + 2] = lo_bf16(hx.y); x[k][8 * v + 3] = hi_bf16(hx.y);
+            x[k][8 * v + 4] = lo_bf16(hx.z); x[k][8 * v + 5] = hi_bf16(hx.z);
+            x[k][8 * v + 6] = lo_bf16(hx.w); x[k][8 * v + 7] = hi_bf16(hx.w);
         }
+    }
+    const uint2 h0 = make_uint2(0, 0);
+    bool ok = true;
+    int flushed = 0;  // rows already reduced and stored
+    // reduce and store rows [flushed, upto) of this CTA; false (the CTA leaves) if any of its
+    // waits gave up. The only CTA-wide barriers: between them the warps run on the ring's
+    // barriers alone, each wait bounded and abandoned as soon as another thread gave up.
+    auto flush = [&](int upto) -> bool {
+        if (__syncthreads_or(!ok)) return false;
+        const int cnt = upto - flushed;
+        if (p.epi >= EMB_EPI_GEGLU) {
+            // gate row 2i and up row 2i + 1 of the CTA (runs start on even rows)
+            if (t < cnt / 2) {
+                float gate = 0.0f, up = 0.0f;
 #pragma unroll
-        for (int r = 0; r < 2; ++r) acc[r] = fmaf(dp[k][r], dot_unit<FMT>(cp[k][r], h0, x), acc[r]);
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            if (r < ns) {
-                const uint4 c = *reinterpret_cast<const uint4*>(codes_s + r * row_bytes + int64_t(uk) * 16);
-                const float d = __half2float(scales_s[r * p.ldS + ((FMT == EMB_Q8_0) ? (uk >> 1) : uk)]);
-                acc[2 + r] = fmaf(d, dot_unit<FMT>(c, h0, x), acc[2 + r]);
+                for (int w = 0; w < NWARP; ++w) {
+                    gate += red[(2 * t) * NWARP + w];
+                    up += red[(2 * t + 1) * NWARP + w];
+                }
+                int g, n;
+                locate(r_begin + flushed + 2 * t, g, n);
+                epi_store_gated(p.epi, p.Y[g], 0, n, p.N[g], gate, up);
             }
+        } else if (t < cnt) {
+            float v = 0.0f;
+#pragma unroll
+            for (int w = 0; w < NWARP; ++w) v += red[t * NWARP + w];
+            int g, n;
+            locate(r_begin + flushed + t, g, n);
+            epi_store(p.epi, p.Y[g], 0, n, p.N[g], v);
         }
-    }
-
-    const int lane = t & 31, warp = t >> 5;
+        __syncthreads();
+        flushed = upto;
+        return true;
+    };
+    // stage and phase of row i, and of row i - 1, kept by increments (no integer division)
+    int s = 0, sp = 0;
+    uint32_t ph = 0, php = 0;
+    for (int i = 0; i < n_rows; ++i) {
+        // refill: the stage of row i - 1 once every warp has released it
+        if (t == 0 && ok && i >= 1 && i - 1 + S < n_rows) {
+            ok = ptx::mbar_wait(&empty[sp], php, abort_flag, p.status, kWaitLimitNs);
+            if (ok) issue(i - 1 + S, sp);
+        }
+        ok = __all_sync(0xffffffffu, ok && ptx::mbar_wait(&full[s], ph, abort_flag, p.status, kWaitLimitNs));
+        if (ok) {
+            const uint8_t* cs = ring + s * p.stage_bytes;
+            const __half* ss = reinterpret_cast<const __half*>(cs + row_bytes);
+            float acc = 0.0f;
 #pragma unroll
-    for (int r = 0; r < 4; ++r) {
-        float v = acc[r];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        if (lane == 0) red[warp * 4 + r] = v;
-    }
-    __syncthreads();
-    if (p.epi >= EMB_EPI_GEGLU) {
-        // gate row row0 + 2i and up row row0 + 2i + 1
-        if (t < 2) {
-            float gate = 0.0f, up = 0.0f;
-#pragma unroll
-            for (int w = 0; w < NWARP; ++w) {
-                gate += red[w * 4 + 2 * t];
-                up += red[w * 4 + 2 * t + 1];
+            for (int k = 0; k < PF; ++k) {
+                const int uk = t + k * NT;
+                if (uk < U) {
+                    const uint4 c = *reinterpret_cast<const uint4*>(cs + int64_t(uk) * 16);
+                    const float d = __half2float(ss[(FMT == EMB_Q8_0) ? (uk >> 1) : uk]);
+                    acc = fmaf(d, dot_unit<FMT>(c, h0, x[k]), acc);
+                }
             }
-            const int n = row0 + 2 * t;
-            if (n < N) epi_store_gated(p.epi, p.Y[g], 0, n, N, gate, up);
-        }
-    } else if (t < 4) {
-        float v = 0.0f;
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&empty[s]);
 #pragma unroll
-        for (int w = 0; w < NWARP; ++w) v += red[w * 4 + t];
-        const int n = row0 + t;
-        if (n < N) epi_store(p.epi, p.Y[g], 0, n, N, v);
+            for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            if (lane == 0) red[(i - flushed) * NWARP + warp] = acc;
+        }
+        if (i + 1 - flushed == kRingFlush && !flush(i + 1)) return;
+        sp = s;
+        php = ph;
+        if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+        }
     }
+    if (flushed < n_rows) flush(n_rows);  // (a CTA whose wait gave up leaves inside it)
 }
 
 template <int FMT, int PF>
-cudaError_t launch_hybrid_one(const HybridParams& p, int tiles, size_t smem, bool pdl, cudaStream_t s) {
+cudaError_t launch_ring_one(const RingParams& p, int ctas, size_t smem, bool pdl, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(tiles, 1, 1);
-    cfg.blockDim = dim3(kHybThreads, 1, 1);
+    cfg.gridDim = dim3(ctas, 1, 1);
+    cfg.blockDim = dim3(kRingThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -1000,38 +1028,51 @@ cudaError_t launch_hybrid_one(const HybridParams& p, int tiles, size_t smem, boo
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
-    if (smem > 48 * 1024) {
-        const cudaError_t e = cudaFuncSetAttribute(gemv_hybrid_kernel<FMT, PF>,
-                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-        if (e != cudaSuccess) return e;
-    }
-    return cudaLaunchKernelEx(&cfg, gemv_hybrid_kernel<FMT, PF>, p);
+    const cudaError_t e = cudaFuncSetAttribute(gemv_ring_kernel<FMT, PF>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    return cudaLaunchKernelEx(&cfg, gemv_ring_kernel<FMT, PF>, p);
 }
 
-// Which layers take the hybrid path: M = 1, Q8_0 or Q4_0, rows longer than the staged path
+int gemv_sm_count() {
+    static std::mutex mu;
+    static int counts[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!counts[dev] && cudaDeviceGetAttribute(&counts[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        counts[dev] = 0;
+    return counts[dev];
+}
+
+// Which layers take the ring path: M = 1, Q8_0 or Q4_0, rows longer than the staged path
 // takes at M = 1 and than one pass of 256 threads (2..4 units per thread), matrices of at
-// least kStageMinBytes. Measured on GB300 (graph-replayed chains of the Gemma-2B down
-// projection, 2048 x 16384, each launch its own weights; register kernel -> hybrid):
-// Q8_0 9.76 -> 9.54 us, Q4_0 9.75 -> 9.65 us.
-bool launch_hybrid(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
+// least kStageMinBytes; two CTAs per SM, rows split evenly (even runs for gated epilogues).
+// Measured on GB300, Gemma-2B decode step (paired runs on one box, 1000 steps): Q8_0 chain
+// 0.507 -> 0.477 ms and Q4_0 0.457 -> 0.455 against a kernel with two rows per CTA in
+// registers and two in shared memory; a 72 KB ring instead of 56 KB was slower for Q8_0,
+// a CTA-wide barrier per row cost ~2 %, and stage indices by integer division ~4 %.
+bool launch_ring(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
     if (g.M != 1 || (g.fmt != EMB_Q8_0 && g.fmt != EMB_Q4_0)) return false;
     const int64_t row_bytes = (g.fmt == EMB_Q8_0) ? g.K : g.K / 2;
     const int64_t U = (g.fmt == EMB_Q8_0) ? g.K / 16 : g.K / 32;
-    if (row_bytes <= kStageMaxRowBytesM1 || U <= kHybThreads || U > 4 * kHybThreads) return false;
+    if (row_bytes <= kStageMaxRowBytesM1 || U <= kRingThreads || U > 4 * kRingThreads) return false;
     int64_t rows = 0;
     for (int i = 0; i < g.n_mats; ++i) rows += g.mats[i].N;
     if (rows * row_bytes < kStageMinBytes) return false;
-    HybridParams p = {};
-    int tiles = 0;
+    const int sms = gemv_sm_count();
+    if (sms <= 0) return false;
+    RingParams p = {};
+    int64_t r0 = 0;
     for (int i = 0; i < g.n_mats; ++i) {
         p.codes[i] = g.mats[i].codes;
         p.scales[i] = g.mats[i].scales;
         p.Y[i] = g.mats[i].Y;
         p.N[i] = int32_t(g.mats[i].N);
-        p.tile0[i] = tiles;
-        tiles += int((g.mats[i].N + 3) / 4);
+        p.row0[i] = int32_t(r0);
+        r0 += g.mats[i].N;
     }
-    p.tile0[g.n_mats] = tiles;
+    p.row0[g.n_mats] = int32_t(r0);
     p.n_mats = g.n_mats;
     p.K = int32_t(g.K);
     p.ldS = int32_t(g.ldS);
@@ -1039,16 +1080,23 @@ bool launch_hybrid(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cud
     p.epi = g.epi;
     p.X = g.X;
     p.status = status;
-    const size_t smem = kHybHeader + size_t(2) * size_t(row_bytes + g.ldS * 2);
-    const int pf = int((U + kHybThreads - 1) / kHybThreads);
+    int64_t rpc = (rows + 2 * sms - 1) / (2 * sms);
+    if (g.epi >= EMB_EPI_GEGLU) rpc = (rpc + 1) & ~int64_t(1);  // gate/up pairs stay in one CTA
+    p.rows_per_cta = int32_t(rpc);
+    p.rows_total = int32_t(rows);
+    p.stage_bytes = int32_t((row_bytes + g.ldS * 2 + 15) & ~int64_t(15));
+    p.stages = int32_t(std::min<int64_t>(kRingMaxStages, std::max<int64_t>(2, kRingBudget / p.stage_bytes)));
+    const int ctas = int((rows + rpc - 1) / rpc);
+    const size_t smem = kRingHeader + size_t(p.stages) * p.stage_bytes;
+    const int pf = int((U + kRingThreads - 1) / kRingThreads);
     if (g.fmt == EMB_Q8_0)
-        err = pf == 2 ? launch_hybrid_one<EMB_Q8_0, 2>(p, tiles, smem, pdl, s)
-            : pf == 3 ? launch_hybrid_one<EMB_Q8_0, 3>(p, tiles, smem, pdl, s)
-                      : launch_hybrid_one<EMB_Q8_0, 4>(p, tiles, smem, pdl, s);
+        err = pf == 2 ? launch_ring_one<EMB_Q8_0, 2>(p, ctas, smem, pdl, s)
+            : pf == 3 ? launch_ring_one<EMB_Q8_0, 3>(p, ctas, smem, pdl, s)
+                      : launch_ring_one<EMB_Q8_0, 4>(p, ctas, smem, pdl, s);
     else
-        err = pf == 2 ? launch_hybrid_one<EMB_Q4_0, 2>(p, tiles, smem, pdl, s)
-            : pf == 3 ? launch_hybrid_one<EMB_Q4_0, 3>(p, tiles, smem, pdl, s)
-                      : launch_hybrid_one<EMB_Q4_0, 4>(p, tiles, smem, pdl, s);
+        err = pf == 2 ? launch_ring_one<EMB_Q4_0, 2>(p, ctas, smem, pdl, s)
+            : pf == 3 ? launch_ring_one<EMB_Q4_0, 3>(p, ctas, smem, pdl, s)
+                      : launch_ring_one<EMB_Q4_0, 4>(p, ctas, smem, pdl, s);
     return true;
 }
 
@@ -1060,7 +1108,7 @@ cudaError_t launch_gemv(const GroupRef& g, bool pdl, int* status, cudaStream_t s
     cudaError_t err = cudaSuccess;
     if (launch_q4_mma(g, pdl, status, s, err)) return err;
     if (launch_staged(g, pdl, status, s, err)) return err;
-    if (launch_hybrid(g, pdl, status, s, err)) return err;
+    if (launch_ring(g, pdl, status, s, err)) return err;
     return launch_gemv_regs(g, pdl, s);
 }
 

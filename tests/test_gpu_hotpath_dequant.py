@@ -179,15 +179,15 @@ GEMV_CASES = [
     # long Q8_0 rows below 12 MB: a thread's whole row share loaded before the wait (PF = 4)
     (emb.EMB_Q8_0, 256, 16384, 1, "register PF=4 R=1", "spread"),
     (emb.EMB_Q6_0, 2048, 16384, 1, "register R=2 long rows", "spread"),
-    # hybrid kernel (rows > 6 KB, >= 12 MB, M = 1): two rows per CTA in registers, two in
-    # shared memory; the Gemma-2B down projection shape, 2..4 units per thread, and ragged
-    # row counts (the last CTA with one or no shared-memory row)
-    (emb.EMB_Q8_0, 2048, 16384, 1, "hybrid PF=4", "spread"),
-    (emb.EMB_Q4_0, 2048, 16384, 1, "hybrid PF=2", "spread"),
-    (emb.EMB_Q8_0, 2048, 8192, 1, "hybrid PF=2", "spread"),
-    (emb.EMB_Q8_0, 1027, 12288, 1, "hybrid PF=3, one smem row in the last CTA", "spread"),
-    (emb.EMB_Q4_0, 1024, 24576, 1, "hybrid PF=3", "spread"),
-    (emb.EMB_Q4_0, 1538, 16384, 1, "hybrid, no smem row in the last CTA", "spread"),
+    # ring kernel (rows > 6 KB, >= 12 MB, M = 1: X in registers, rows through a shared-memory
+    # ring): the Gemma-2B down projection shape, 2..4 units per thread, ragged last CTAs
+    (emb.EMB_Q8_0, 2048, 16384, 1, "ring PF=4", "spread"),
+    (emb.EMB_Q8_0, 2048, 8192, 1, "ring PF=2", "spread"),
+    (emb.EMB_Q8_0, 1027, 12288, 1, "ring PF=3, ragged last CTA", "spread"),
+    (emb.EMB_Q4_0, 2048, 16384, 1, "ring PF=2", "spread"),
+    (emb.EMB_Q4_0, 1024, 24576, 1, "ring PF=3", "spread"),
+    (emb.EMB_Q4_0, 1538, 16384, 1, "ring, ragged last CTA", "spread"),
+    (emb.EMB_Q4_0, 1539, 16384, 1, "ring, ragged last CTA", "spread"),
     # staged kernel: >= 12 MB of codes with rows <= 6 KB at M = 1; any rows at M = 2..4
     (emb.EMB_Q8_0, 6144, 2048, 1, "staged", "all"),
     (emb.EMB_Q8_0, 6144, 2048, 4, "staged MT=4", "all"),

@@ -52,6 +52,29 @@ def test_seq_equals_single_calls_and_oracle(cuda_device, fmt, M):
         check_close(seq_out[i].cpu().numpy(), Yref, B, f"layer {i}")
 
 
+@pytest.mark.parametrize("fmt", [emb.EMB_Q8_0, emb.EMB_Q4_0])
+def test_long_rows_group_across_matrices(cuda_device, fmt):
+    """Two long-row matrices sharing X at M = 1 form one launch of the ring kernel, whose
+    CTAs own runs of rows that cross from the first matrix into the second: bitwise the
+    separate calls, within the oracle's bound."""
+    K, Ns, M = 16384, (1000, 1030), 1
+    Xb = activation_bits_np(M, K, 77)
+    X = to_dev_bf16(Xb)
+    Ws = [weight_np(N, K, 78 + i) for i, N in enumerate(Ns)]
+    imgs = [emb.quantize(fmt, torch.from_numpy(W).cuda()) for W in Ws]
+    Ys = [torch.full((M, N), float("nan"), device="cuda") for N in Ns]
+    emb.emb_qlayer_seq([(fmt, img, N, K, X, Y) for img, N, Y in zip(imgs, Ns, Ys)], M)
+    torch.cuda.synchronize()
+    for img, N, Y, W in zip(imgs, Ns, Ys, Ws):
+        Y1 = torch.full_like(Y, float("nan"))
+        emb.emb_qmatmul(fmt, img, X, Y1, M, N, K)
+        torch.cuda.synchronize()
+        assert torch.equal(Y.view(torch.int32), Y1.view(torch.int32)), N
+        Yref, B = oracle.qmatmul(fmt, oracle.quantize(fmt, W), Xb, N, K)
+        check_close(Y.cpu().numpy(), Yref, B, f"fmt={fmt} N={N}")
+    assert emb.emb_device_status() == emb.EMB_OK
+
+
 @pytest.mark.parametrize("M", [1, 50])
 def test_seq_graph_replay(cuda_device, M):
     fmt = emb.EMB_Q8_0
