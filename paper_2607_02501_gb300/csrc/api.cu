@@ -546,7 +546,7 @@ const char* emb_status_string(emb_status status) {
 }
 
 const char* emb_build_info(void) {
-    return "libembqmm: sm_103a; Q8_0/Q6_0/Q4_0; GEMV (M<=4: staged/register FFMA2, Q4_0 mma.sync at M>=2) + "
+    return "libembqmm: sm_103a; Q8_0/Q6_0/Q4_0; GEMV (M<=4: staged/ring/register FFMA2, Q4_0 mma.sync at M>=2) + "
            "tcgen05 GEMM (M>4: TMA, dequant to bf16 A tiles in TMEM, TMEM accumulators; one tile, persistent, "
            "cluster split-K or stream-K schedules); "
            "recorded chains (CUDA graphs); RMSNorm, rotary embedding, grouped-head attention";
