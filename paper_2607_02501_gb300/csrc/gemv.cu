@@ -865,6 +865,7 @@ constexpr int kRingHeader = 144 + kRingFlush * (kRingThreads / 32) * 4;
 
 struct RingParams {
     const uint8_t* codes[kMaxGroup];
+    const uint8_t* high[kMaxGroup];  // Q6_0: 2-bit high plane of each matrix
     const __half* scales[kMaxGroup];
     void* Y[kMaxGroup];
     int32_t N[kMaxGroup];
@@ -872,7 +873,7 @@ struct RingParams {
     int32_t n_mats;
     int32_t K, ldS, U;
     int32_t rows_per_cta, rows_total;
-    int32_t stage_bytes;          // one row of codes + its scales, rounded up to 16
+    int32_t stage_bytes;          // one row of codes (+ Q6_0 high bits) + its scales, rounded up to 16
     int32_t stages;               // ring depth (2..kRingMaxStages)
     int32_t epi;
     const __nv_bfloat16* X;
@@ -893,6 +894,7 @@ __global__ void __launch_bounds__(kRingThreads, 2) gemv_ring_kernel(const __grid
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int U = p.U;
     const int64_t row_bytes = (FMT == EMB_Q8_0) ? int64_t(p.K) : int64_t(p.K) / 2;
+    const int64_t high_bytes = (FMT == EMB_Q6_0) ? int64_t(p.K) / 4 : 0;  // a multiple of 16
     const int r_begin = blockIdx.x * p.rows_per_cta;
     const int n_rows = min(p.rows_per_cta, p.rows_total - r_begin);
     // global row -> (matrix, row within it)
@@ -908,10 +910,11 @@ __global__ void __launch_bounds__(kRingThreads, 2) gemv_ring_kernel(const __grid
         locate(r_begin + i, g, n);
         uint8_t* st = ring + stage * p.stage_bytes;
         uint64_t* bar = &full[stage];
-        const uint32_t cb = uint32_t(row_bytes), sb = uint32_t(p.ldS) * 2u;
-        ptx::mbar_arrive_expect_tx(bar, cb + sb);
+        const uint32_t cb = uint32_t(row_bytes), hb = uint32_t(high_bytes), sb = uint32_t(p.ldS) * 2u;
+        ptx::mbar_arrive_expect_tx(bar, cb + hb + sb);
         ptx::bulk_load(st, p.codes[g] + int64_t(n) * row_bytes, cb, bar);
-        ptx::bulk_load(st + row_bytes, p.scales[g] + int64_t(n) * p.ldS, sb, bar);
+        if constexpr (FMT == EMB_Q6_0) ptx::bulk_load(st + row_bytes, p.high[g] + int64_t(n) * high_bytes, hb, bar);
+        ptx::bulk_load(st + row_bytes + high_bytes, p.scales[g] + int64_t(n) * p.ldS, sb, bar);
     };
     if (t == 0) {
         *abort_flag = 0;
@@ -988,15 +991,17 @@ __global__ void __launch_bounds__(kRingThreads, 2) gemv_ring_kernel(const __grid
         ok = __all_sync(0xffffffffu, ok && ptx::mbar_wait(&full[s], ph, abort_flag, p.status, kWaitLimitNs));
         if (ok) {
             const uint8_t* cs = ring + s * p.stage_bytes;
-            const __half* ss = reinterpret_cast<const __half*>(cs + row_bytes);
+            const __half* ss = reinterpret_cast<const __half*>(cs + row_bytes + high_bytes);
             float acc = 0.0f;
 #pragma unroll
             for (int k = 0; k < PF; ++k) {
                 const int uk = t + k * NT;
                 if (uk < U) {
                     const uint4 c = *reinterpret_cast<const uint4*>(cs + int64_t(uk) * 16);
+                    uint2 hq = h0;
+                    if constexpr (FMT == EMB_Q6_0) hq = *reinterpret_cast<const uint2*>(cs + row_bytes + int64_t(uk) * 8);
                     const float d = __half2float(ss[(FMT == EMB_Q8_0) ? (uk >> 1) : uk]);
-                    acc = fmaf(d, dot_unit<FMT>(c, h0, x[k]), acc);
+                    acc = fmaf(d, dot_unit<FMT>(c, hq, x[k]), acc);
                 }
             }
             __syncwarp();
@@ -1045,27 +1050,30 @@ int gemv_sm_count() {
     return counts[dev];
 }
 
-// Which layers take the ring path: M = 1, Q8_0 or Q4_0, rows longer than the staged path
-// takes at M = 1 and than one pass of 256 threads (2..4 units per thread), matrices of at
-// least kStageMinBytes; two CTAs per SM, rows split evenly (even runs for gated epilogues).
+// Which layers take the ring path: M = 1, Q8_0, Q4_0 or Q6_0 (K % 64 == 0, for its high
+// plane's 16-byte rows), rows longer than the staged path takes at M = 1 and than one pass
+// of 256 threads (2..4 units per thread), matrices of at least kStageMinBytes; two CTAs per
+// SM, rows split evenly (even runs for gated epilogues).
 // Measured on GB300, Gemma-2B decode step (paired runs on one box, 1000 steps): Q8_0 chain
 // 0.507 -> 0.477 ms and Q4_0 0.457 -> 0.455 against a kernel with two rows per CTA in
 // registers and two in shared memory; a 72 KB ring instead of 56 KB was slower for Q8_0,
 // a CTA-wide barrier per row cost ~2 %, and stage indices by integer division ~4 %.
 bool launch_ring(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaError_t& err) {
-    if (g.M != 1 || (g.fmt != EMB_Q8_0 && g.fmt != EMB_Q4_0)) return false;
+    if (g.M != 1 || (g.fmt == EMB_Q6_0 && g.K % 64 != 0)) return false;
     const int64_t row_bytes = (g.fmt == EMB_Q8_0) ? g.K : g.K / 2;
+    const int64_t high_bytes = (g.fmt == EMB_Q6_0) ? g.K / 4 : 0;
     const int64_t U = (g.fmt == EMB_Q8_0) ? g.K / 16 : g.K / 32;
-    if (row_bytes <= kStageMaxRowBytesM1 || U <= kRingThreads || U > 4 * kRingThreads) return false;
+    if (row_bytes + high_bytes <= kStageMaxRowBytesM1 || U <= kRingThreads || U > 4 * kRingThreads) return false;
     int64_t rows = 0;
     for (int i = 0; i < g.n_mats; ++i) rows += g.mats[i].N;
-    if (rows * row_bytes < kStageMinBytes) return false;
+    if (rows * (row_bytes + high_bytes) < kStageMinBytes) return false;
     const int sms = gemv_sm_count();
     if (sms <= 0) return false;
     RingParams p = {};
     int64_t r0 = 0;
     for (int i = 0; i < g.n_mats; ++i) {
         p.codes[i] = g.mats[i].codes;
+        p.high[i] = g.mats[i].high;
         p.scales[i] = g.mats[i].scales;
         p.Y[i] = g.mats[i].Y;
         p.N[i] = int32_t(g.mats[i].N);
@@ -1084,7 +1092,7 @@ bool launch_ring(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaE
     if (g.epi >= EMB_EPI_GEGLU) rpc = (rpc + 1) & ~int64_t(1);  // gate/up pairs stay in one CTA
     p.rows_per_cta = int32_t(rpc);
     p.rows_total = int32_t(rows);
-    p.stage_bytes = int32_t((row_bytes + g.ldS * 2 + 15) & ~int64_t(15));
+    p.stage_bytes = int32_t((row_bytes + high_bytes + g.ldS * 2 + 15) & ~int64_t(15));
     p.stages = int32_t(std::min<int64_t>(kRingMaxStages, std::max<int64_t>(2, kRingBudget / p.stage_bytes)));
     const int ctas = int((rows + rpc - 1) / rpc);
     const size_t smem = kRingHeader + size_t(p.stages) * p.stage_bytes;
@@ -1093,10 +1101,14 @@ bool launch_ring(const GroupRef& g, bool pdl, int* status, cudaStream_t s, cudaE
         err = pf == 2 ? launch_ring_one<EMB_Q8_0, 2>(p, ctas, smem, pdl, s)
             : pf == 3 ? launch_ring_one<EMB_Q8_0, 3>(p, ctas, smem, pdl, s)
                       : launch_ring_one<EMB_Q8_0, 4>(p, ctas, smem, pdl, s);
-    else
+    else if (g.fmt == EMB_Q4_0)
         err = pf == 2 ? launch_ring_one<EMB_Q4_0, 2>(p, ctas, smem, pdl, s)
             : pf == 3 ? launch_ring_one<EMB_Q4_0, 3>(p, ctas, smem, pdl, s)
                       : launch_ring_one<EMB_Q4_0, 4>(p, ctas, smem, pdl, s);
+    else
+        err = pf == 2 ? launch_ring_one<EMB_Q6_0, 2>(p, ctas, smem, pdl, s)
+            : pf == 3 ? launch_ring_one<EMB_Q6_0, 3>(p, ctas, smem, pdl, s)
+                      : launch_ring_one<EMB_Q6_0, 4>(p, ctas, smem, pdl, s);
     return true;
 }
 

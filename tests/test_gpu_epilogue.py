@@ -56,11 +56,12 @@ def run_epilogue(fmt, kind, M, N, K, seed):
 # GEMM one token tile per CTA, GEMM two token tiles per CTA, Q6_0 GEMV and GEMM, Q8_0
 # register GEMV loading whole row shares before the wait (long rows, two rows per CTA), Q4_0
 # staged GEMV at M = 1 with a ragged last tile, GEMM with persistent CTAs (320 tiles), the
-# ring GEMV (long rows, >= 12 MB, M = 1; the second with a ragged last CTA)
+# ring GEMV (long rows, >= 12 MB, M = 1; the second and third with a ragged last CTA, the
+# third with the Q6_0 high plane)
 PATHS = [(Q8, 1, 256, 1024), (Q8, 1, 24576, 2048), (Q4, 4, 600, 2080), (Q4, 4, 32768, 1024),
          (Q8, 64, 384, 320), (Q8, 50, 1000, 1024), (Q4, 136, 640, 2048), (Q8, 280, 11008, 1024),
          (Q6, 1, 4096, 2048), (Q6, 50, 512, 2048), (Q8, 1, 1300, 7168), (Q4, 1, 16392, 2048),
-         (Q8, 816, 10240, 1024), (Q8, 1, 2048, 16384), (Q4, 1, 1538, 16384)]
+         (Q8, 816, 10240, 1024), (Q8, 1, 2048, 16384), (Q4, 1, 1538, 16384), (Q6, 1, 1026, 16384)]
 
 
 @pytest.mark.parametrize("kind", KINDS)

@@ -178,7 +178,8 @@ GEMV_CASES = [
     (emb.EMB_Q8_0, 2048, 2048, 2, "register R=4 MT=2", "all"),
     # long Q8_0 rows below 12 MB: a thread's whole row share loaded before the wait (PF = 4)
     (emb.EMB_Q8_0, 256, 16384, 1, "register PF=4 R=1", "spread"),
-    (emb.EMB_Q6_0, 2048, 16384, 1, "register R=2 long rows", "spread"),
+    (emb.EMB_Q6_0, 1024, 8192, 1, "register R=2 long rows (< 12 MB)", "spread"),
+    (emb.EMB_Q6_0, 2048, 16384, 1, "ring, Q6_0 high plane in the stage", "spread"),
     # ring kernel (rows > 6 KB, >= 12 MB, M = 1: X in registers, rows through a shared-memory
     # ring): the Gemma-2B down projection shape, 2..4 units per thread, ragged last CTAs
     (emb.EMB_Q8_0, 2048, 16384, 1, "ring PF=4", "spread"),
